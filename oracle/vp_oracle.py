@@ -1,0 +1,249 @@
+"""CPU oracle for one VisionPulse decode step (test infrastructure only).
+
+This module is test infrastructure.  Only ``tests/``, ``__graft_entry__.smoke()``
+and ``bench.py`` (its ``cpu_baseline`` leg and its ``--impl reference`` arm)
+may import it.  The library path (``libvp.so`` and its Python binding) never
+imports, links or runs anything here, and this module imports nothing from the
+library: the two share no code.
+
+What it computes, for one attention layer acting as the anchor layer l_a and
+one decode step t (VisionPulse, Sec. 4.2-4.3 and Sec. 5.2):
+
+  1. pre-softmax logits  Z_{t,h}(q_t, j) = scale * <q_h, k_j>     (Eq. 6's Z)
+  2. attention probabilities at tau = 1 and at tau                  (Eq. 6)
+     -- both normalised over EVERY cached token j (visual and text)
+  3. per-head visual mass m_{t,h}, its head mean M_vis and the
+     head-max M_vis,max                                             (Eq. 5, Sec. 4.3)
+  4. the retention budget K_t = M_vis,max * N_v, clamped            (Eq. 7, Sec. 5.2)
+  5. importance S_i = (1/H) sum_h A_{t,h}(q_t, v_i)                  (Eq. 2)
+  6. X_v^t = Top-K_t(S)                                              (Eq. 3)
+  7. attention of q_t over X_v^t plus all text tokens               (Sec. 4.2, Sec. 5.7)
+
+Everything is float64 computed from the exact input values (bf16 or fp32
+inputs are widened without rounding).  There is no blocking, fusion or
+reordering beyond the definitions above.
+
+Readings of points the paper leaves open (each is listed in the design doc):
+  * Eq. 2 uses the plain softmax (tau = 1); tau enters only the mass (Eq. 6).
+  * H is the number of query heads; under grouped-query attention query head h
+    reads kv-head h // G with G = H / Hkv.
+  * The softmax normaliser of Eq. 6 runs over all cached tokens (visual, text
+    and the current token); a visual-only normaliser would make the mass 1.
+  * K_t = ceil(M_vis,max * N_v) with the product and the ceiling taken in
+    float32 (the kernel's precision, since a float decides an integer here);
+    clamp [K_lo, K_hi] with K_lo = ceil(r_lo N_v), K_hi = max(K_lo, floor(r_hi N_v)),
+    ratios given in parts per million and multiplied in exact integers.
+  * Top-K ranks S_i rounded to float32 (the kernel's precision); equal keys
+    go to the lower visual index.  Indices are returned ascending and relative
+    to the start of the visual span.
+  * granularity 1 ("per kv-head") averages S over the G query heads of each
+    kv-head only and keeps K_t (from the head-max over all H heads) per kv-head.
+"""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+# Budget modes (same numbering as the C header, restated here so that the
+# oracle depends on nothing in the library).
+ADAPTIVE = 0      # Eq. 7 with the clamp of Sec. 5.2
+FIXED_RATIO = 1   # "FastV-VP (Fix Ratio)", Sec. 5.4 / Table 2
+FIXED_K = 2       # constant Top-k budget, App. A.2
+DENSE = 3         # keep every visual token (full budget)
+
+PPM = 1_000_000
+
+
+def logits(q: np.ndarray, k: np.ndarray, scale: float) -> np.ndarray:
+    """Pre-softmax attention logits Z_{t,h}(q_t, j) (the Z of Eq. 6, Sec. 4.3).
+
+    q: [H, D] query of the current token, k: [Hkv, T, D] cached keys.
+    Query head h reads kv-head h // G (grouped-query attention, G = H / Hkv).
+    Returns z: [H, T], z[h, j] = scale * <q[h], k[h // G, j]>.
+    """
+    H = q.shape[0]
+    Hkv = k.shape[0]
+    G = H // Hkv
+    z = np.empty((H, k.shape[1]), dtype=np.float64)
+    for h in range(H):
+        z[h] = scale * (k[h // G].astype(np.float64) @ q[h].astype(np.float64))
+    return z
+
+
+def softmax_tau(z: np.ndarray, tau: float) -> np.ndarray:
+    """Temperature-scaled attention probabilities A^{(tau)} of Eq. 6 (Sec. 4.3).
+
+    A^{(tau)}_{h}(j) = exp(Z_h(j) / tau) / sum_{j'} exp(Z_h(j') / tau), the sum
+    running over every cached token j' of the row.  tau = 1 gives the plain
+    attention probability A of Eq. 2.  The row maximum is subtracted first;
+    this changes nothing mathematically.
+    """
+    m = z.max(axis=-1, keepdims=True)
+    e = np.exp((z - m) / tau)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def visual_mass(a_tau: np.ndarray, vis: np.ndarray):
+    """Visual attention mass, Eq. 5 and the head-max variant of Sec. 4.3.
+
+    a_tau: [H, T] probabilities, vis: boolean [T] marking the visual span.
+    Returns (m [H], M_vis = mean_h m, M_vis,max = max_h m).  With no visual
+    token every m is 0.
+    """
+    m = a_tau[:, vis].sum(axis=1) if vis.any() else np.zeros(a_tau.shape[0])
+    return m, float(m.mean()), float(m.max())
+
+
+def _ceil_div(a: int, b: int) -> int:
+    return -((-a) // b)
+
+
+def budget_bounds(n_v: int, r_lo_ppm: int, r_hi_ppm: int):
+    """Clamp range of Sec. 5.2, "(0.01N, 0.05N)" read as [K_lo, K_hi].
+
+    K_lo = ceil(r_lo * N_v), K_hi = max(K_lo, floor(r_hi * N_v)), with the
+    ratios in parts per million and the products in exact integers.
+    """
+    k_lo = _ceil_div(r_lo_ppm * n_v, PPM)
+    k_hi = max(k_lo, (r_hi_ppm * n_v) // PPM)
+    return k_lo, k_hi
+
+
+def budget(m_max: float, n_v: int, mode: int = ADAPTIVE, r_lo_ppm: int = 10_000,
+           r_hi_ppm: int = 50_000, ratio_ppm: int = 0, fixed_k: int = 0) -> int:
+    """Step-wise retention budget K_t.
+
+    ADAPTIVE    : K_t = M_vis,max * N_v (Eq. 7), rounded up, clamped to
+                  [K_lo, K_hi] (Sec. 5.2).  The float32 product and ceiling
+                  mirror the precision in which the kernel takes the decision.
+    FIXED_RATIO : K_t = ceil(r * N_v), at least 1 ("Fix Ratio", Table 2).
+    FIXED_K     : K_t = min(k, N_v) (Top-k budgeting, App. A.2).
+    DENSE       : K_t = N_v.
+    N_v = 0 gives K_t = 0 in every mode.
+    """
+    if n_v <= 0:
+        return 0
+    if mode == DENSE:
+        return n_v
+    if mode == FIXED_K:
+        return max(0, min(int(fixed_k), n_v))
+    if mode == FIXED_RATIO:
+        return min(max(_ceil_div(ratio_ppm * n_v, PPM), 1), n_v)
+    if mode != ADAPTIVE:
+        raise ValueError(f"unknown budget mode {mode}")
+    prod = np.float32(m_max) * np.float32(n_v)          # float32 product
+    raw = int(math.ceil(float(prod)))
+    k_lo, k_hi = budget_bounds(n_v, r_lo_ppm, r_hi_ppm)
+    return min(max(raw, k_lo), k_hi, n_v)
+
+
+def importance(a: np.ndarray, vis: np.ndarray, heads=None) -> np.ndarray:
+    """Importance score of Eq. 2: S_i = (1/H) sum_h A_h(q_t, v_i) over visual i.
+
+    a: [H, T] plain (tau = 1) probabilities.  ``heads`` restricts the average
+    to a subset of query heads (the per-kv-head reading); None = all H heads.
+    """
+    rows = a if heads is None else a[list(heads)]
+    return rows[:, vis].mean(axis=0)
+
+
+def select_topk(s: np.ndarray, k: int) -> np.ndarray:
+    """X_v^t = Top-K_t(S), Eq. 3.  Largest scores first, ties to the lower index.
+
+    Scores are ranked as float32 values (the precision the kernel decides in).
+    Returns the kept visual indices in ascending order.
+    """
+    key = np.asarray(s, dtype=np.float32)
+    order = sorted(range(len(key)), key=lambda i: (-float(key[i]), i))
+    return np.array(sorted(order[:k]), dtype=np.int64)
+
+
+def pruned_attention(z: np.ndarray, v: np.ndarray, keep: np.ndarray) -> np.ndarray:
+    """Attention output over the kept tokens only (Sec. 4.2; the "dynamic
+    visual sparse attention" of Sec. 5.7).
+
+    z: [H, T] logits, v: [Hkv, T, D] values, keep: boolean [T] (kept visual
+    tokens plus every text token).  Dropped tokens are excluded from the
+    softmax, not given weight zero inside a larger normaliser:
+        out_h = sum_{j in keep} exp(z_hj) v_j / sum_{j in keep} exp(z_hj).
+    """
+    H = z.shape[0]
+    G = H // v.shape[0]
+    out = np.empty((H, v.shape[2]), dtype=np.float64)
+    for h in range(H):
+        zk = z[h, keep]
+        w = np.exp(zk - zk.max())
+        out[h] = (w @ v[h // G][keep].astype(np.float64)) / w.sum()
+    return out
+
+
+def decode_step(q, k, v, vis_start: int, vis_len: int, text_len: int, *,
+                mode: int = ADAPTIVE, tau: float = 0.1, scale: float = 0.0,
+                r_lo_ppm: int = 10_000, r_hi_ppm: int = 50_000, ratio_ppm: int = 0,
+                fixed_k: int = 0, granularity: int = 0, force_k=None) -> dict:
+    """One VisionPulse decode step for one sequence at the anchor layer.
+
+    q: [H, D]; k, v: [Hkv, >=T, D] with T = vis_len + text_len live tokens.
+    Visual tokens occupy [vis_start, vis_start + vis_len); every other live
+    token (prompt, generated reasoning, current token) is text.
+    ``force_k`` overrides the budget (used by tests to re-select with the
+    other side's K_t near an integer boundary).
+
+    Returns a dict with
+      out [H, D] float64, k_t int, kept list of index arrays (one per sequence
+      for granularity 0, one per kv-head for granularity 1), mass [H]
+      (tau-mass per head), mass_stats [M_vis(tau), M_vis,max(tau),
+      M_vis(tau=1), K_t], z [H, T], s (importance, [N_v] or [Hkv, N_v]).
+    """
+    q = np.asarray(q, dtype=np.float64)
+    H, D = q.shape
+    Hkv = k.shape[0]
+    G = H // Hkv
+    T = vis_len + text_len
+    if text_len < 1:
+        raise ValueError("text_len must count at least the current token")
+    if not (0 <= vis_start <= text_len):
+        raise ValueError("visual span must lie inside the live cache")
+    if scale == 0.0:
+        scale = 1.0 / math.sqrt(D)
+    k = np.asarray(k[:, :T], dtype=np.float64)
+    v = np.asarray(v[:, :T], dtype=np.float64)
+    vis = np.zeros(T, dtype=bool)
+    vis[vis_start:vis_start + vis_len] = True
+
+    z = logits(q, k, scale)                                  # Eq. 6's Z
+    a1 = softmax_tau(z, 1.0)                                 # Eq. 2's A
+    a_tau = softmax_tau(z, tau)                              # Eq. 6
+    mass, m_mean, m_max = visual_mass(a_tau, vis)            # Eq. 5 + head-max
+    _, m_mean1, _ = visual_mass(a1, vis)
+    k_t = budget(m_max, vis_len, mode, r_lo_ppm, r_hi_ppm, ratio_ppm, fixed_k)
+    if force_k is not None:
+        k_t = int(force_k)
+
+    if granularity == 0:
+        s = importance(a1, vis)                              # Eq. 2
+        kept = [select_topk(s, k_t)]                         # Eq. 3
+        out = _attend(z, v, vis_start, vis, kept, G, per_head=False)
+    else:
+        s = np.stack([importance(a1, vis, range(g * G, (g + 1) * G)) for g in range(Hkv)])
+        kept = [select_topk(s[g], k_t) for g in range(Hkv)]
+        out = _attend(z, v, vis_start, vis, kept, G, per_head=True)
+
+    return dict(out=out, k_t=k_t, kept=kept, mass=mass,
+                mass_stats=np.array([m_mean, m_max, m_mean1, float(k_t)]),
+                z=z, s=s)
+
+
+def _attend(z, v, vis_start, vis, kept, G, per_head):
+    """Pruned attention with the kept set(s); text tokens are always kept."""
+    H = z.shape[0]
+    out = np.empty((H, v.shape[2]), dtype=np.float64)
+    for h in range(H):
+        sel = kept[h // G] if per_head else kept[0]
+        keep = ~vis
+        keep[vis_start + sel] = True
+        out[h] = pruned_attention(z[h:h + 1], v[h // G:h // G + 1], keep)[0]
+    return out
+

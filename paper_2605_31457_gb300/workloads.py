@@ -1,0 +1,253 @@
+"""Seeded synthetic inputs for the VisionPulse decode step.
+
+This module only draws inputs: cached keys/values, queries, visual spans,
+text lengths and (optionally) a shuffled paged layout.  It holds none of the
+method's arithmetic (no logits, softmax, mass, budget or selection), so both
+the CUDA path and the CPU oracle may consume what it produces.  Everything is
+drawn on the host with numpy from a fixed seed, then rounded once to the cache
+dtype; the oracle widens those exact values and the GPU reads the same bytes.
+
+Recipe (the same for every workload, with per-workload knobs):
+  * keys, values and query noise are iid N(0, 1);
+  * per (layer, sequence, kv-head) and focus group f, a unit "focus" vector
+    u_f; a fraction ``planted_frac`` of the visual positions get keys
+    sqrt(D) * (0.8 u_f + 0.6 w) with w a unit vector orthogonal to u_f
+    (cosine 0.8 with the focus direction);
+  * optionally a text "sink" key sqrt(D) * u_s at the first text position
+    (a token every query attends to, giving a low visual-mass floor);
+  * the query of head h at step s is
+        sqrt(D) * (beta_v * u_f(s) + beta_s * u_s) + N(0, I),
+    with beta_v drawn log-uniformly per (step, sequence, head) from
+    ``beta_range`` (scaled per sequence by ``seq_beta``) and the focus group
+    f(s) changing every ``focus_every`` steps (shifting visual focus);
+  * optionally every key row is multiplied by a lognormal(0, key_sigma)
+    factor (heavy-tailed key norms).
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field, replace
+
+import numpy as np
+
+BF16 = "bf16"
+FP32 = "fp32"
+
+
+@dataclass(frozen=True)
+class Recipe:
+    name: str
+    layers: int
+    batch: int
+    heads: int
+    kv_heads: int
+    head_dim: int
+    dtype: str
+    vis_len: tuple            # per sequence (len == batch) or a single value
+    vis_start: tuple          # prompt tokens before the visual span, per sequence
+    text_len: tuple           # text tokens at step 0, including the current token
+    steps: int
+    planted_frac: float
+    seed: int
+    n_focus: int = 1
+    focus_every: int = 0      # 0 = never change focus
+    beta_range: tuple = (1.0, 1.0)
+    seq_beta: tuple = ()      # optional per-sequence multiplier of beta_v
+    beta_sink: float = 0.0    # 0 = no sink token
+    key_sigma: float = 0.0    # lognormal sigma of key norms (0 = off)
+    paged: bool = False
+    page_size: int = 16
+    budget: dict = field(default_factory=dict)
+
+    def per_seq(self, v):
+        v = tuple(v) if isinstance(v, (tuple, list)) else (v,)
+        return np.array(v * self.batch if len(v) == 1 else v, dtype=np.int32)
+
+    @property
+    def vis_lens(self):
+        return self.per_seq(self.vis_len)
+
+    @property
+    def vis_starts(self):
+        return self.per_seq(self.vis_start)
+
+    @property
+    def text_lens(self):
+        return self.per_seq(self.text_len)
+
+    def capacity(self, steps=None):
+        """Token capacity of the per-sequence cache for ``steps`` decode steps."""
+        steps = self.steps if steps is None else steps
+        return int((self.vis_lens + self.text_lens).max()) + max(steps - 1, 0)
+
+
+def _rng(seed, *tags):
+    return np.random.default_rng([int(seed)] + [int(t) for t in tags])
+
+
+def _unit(rng, shape):
+    x = rng.standard_normal(shape)
+    return x / np.linalg.norm(x, axis=-1, keepdims=True)
+
+
+def _orth_unit(rng, u):
+    """Unit vectors orthogonal to the unit vectors u (same leading shape)."""
+    w = rng.standard_normal(u.shape)
+    w -= (w * u).sum(-1, keepdims=True) * u
+    return w / np.linalg.norm(w, axis=-1, keepdims=True)
+
+
+@dataclass
+class LayerInputs:
+    k: np.ndarray            # [B, Hkv, Tcap, D] float32 (before dtype rounding)
+    v: np.ndarray            # [B, Hkv, Tcap, D]
+    focus: np.ndarray        # [n_focus, B, Hkv, D] unit
+    sink_dir: np.ndarray     # [B, Hkv, D] unit
+    planted: list            # planted[f][b] -> visual-relative positions
+
+
+def make_layer(r: Recipe, layer: int, t_cap: int | None = None) -> LayerInputs:
+    """Keys and values of one layer's cache for every sequence of the batch."""
+    B, Hkv, D = r.batch, r.kv_heads, r.head_dim
+    t_cap = r.capacity() if t_cap is None else t_cap
+    rng = _rng(r.seed, layer, 1)
+    k = rng.standard_normal((B, Hkv, t_cap, D), dtype=np.float32)
+    v = rng.standard_normal((B, Hkv, t_cap, D), dtype=np.float32)
+    focus = _unit(rng, (r.n_focus, B, Hkv, D))
+    sink_dir = _orth_unit(rng, focus[0])
+    sqd = math.sqrt(D)
+    vis_starts, vis_lens, text_lens = r.vis_starts, r.vis_lens, r.text_lens
+    planted = []
+    for f in range(r.n_focus):
+        pf = []
+        for b in range(B):
+            nv = int(vis_lens[b])
+            n_p = min(nv, int(round(r.planted_frac * nv)))
+            pos = np.sort(rng.choice(nv, size=n_p, replace=False)) if n_p else np.zeros(0, np.int64)
+            pf.append(pos)
+            if n_p:
+                u = np.broadcast_to(focus[f, b][:, None, :], (Hkv, n_p, D))
+                w = _orth_unit(rng, np.ascontiguousarray(u))
+                k[b, :, vis_starts[b] + pos, :] = np.transpose(sqd * (0.8 * u + 0.6 * w), (1, 0, 2))
+        planted.append(pf)
+    if r.beta_sink > 0:
+        for b in range(B):
+            first_text = 0 if vis_starts[b] > 0 else int(vis_lens[b])
+            k[b, :, first_text, :] = sqd * sink_dir[b]
+    if r.key_sigma > 0:
+        k *= np.exp(r.key_sigma * rng.standard_normal((B, Hkv, t_cap, 1))).astype(np.float32)
+    return LayerInputs(k=k, v=v, focus=focus, sink_dir=sink_dir, planted=planted)
+
+
+def make_queries(r: Recipe, layer: int, li: LayerInputs, steps: int | None = None) -> np.ndarray:
+    """Queries [steps, B, H, D] float32 of one layer for ``steps`` decode steps."""
+    steps = r.steps if steps is None else steps
+    B, H, Hkv, D = r.batch, r.heads, r.kv_heads, r.head_dim
+    G = H // Hkv
+    rng = _rng(r.seed, layer, 2)
+    lo, hi = r.beta_range
+    beta = np.exp(rng.uniform(math.log(lo), math.log(hi), size=(steps, B, H)))
+    if r.seq_beta:
+        beta = beta * np.asarray(r.seq_beta, dtype=np.float64)[None, :, None]
+    noise = rng.standard_normal((steps, B, H, D))
+    fidx = np.zeros(steps, dtype=np.int64)
+    if r.focus_every > 0:
+        fidx = (np.arange(steps) // r.focus_every) % r.n_focus
+    u = li.focus[fidx]                                     # [steps, B, Hkv, D]
+    u = np.repeat(u, G, axis=2)                            # [steps, B, H, D]
+    us = np.repeat(li.sink_dir, G, axis=1)[None]           # [1, B, H, D]
+    q = math.sqrt(D) * (beta[..., None] * u + r.beta_sink * us) + noise
+    return q.astype(np.float32)
+
+
+def round_to(x: np.ndarray, dtype: str):
+    """Round float32 values once to the cache dtype; returns a CPU torch tensor."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(x))
+    return t.to(torch.bfloat16) if dtype == BF16 else t.to(torch.float32)
+
+
+def page_table(batch: int, t_cap: int, page_size: int, seed: int, extra_pages: int = 3):
+    """A shuffled page assignment for a paged cache of ``batch`` sequences.
+
+    Returns (block_table [batch, max_pages] int32, n_pages, max_pages): logical
+    page p of sequence b lives in pool page block_table[b, p]; a few pool pages
+    are left unused.
+    """
+    max_pages = -(-t_cap // page_size)
+    n_pages = batch * max_pages + extra_pages
+    perm = _rng(seed, 7).permutation(n_pages)[: batch * max_pages].reshape(batch, max_pages)
+    return perm.astype(np.int32), n_pages, max_pages
+
+
+def scatter_pages(x, block_table, n_pages, page_size):
+    """Copy a contiguous cache into the pool described by ``block_table``."""
+    import torch
+    B, Hkv, T, D = x.shape
+    max_pages = block_table.shape[1]
+    pad = max_pages * page_size - T
+    xt = torch.as_tensor(x)
+    if pad:
+        xt = torch.cat([xt, xt.new_zeros(B, Hkv, pad, D)], dim=2)
+    pool = xt.new_zeros(n_pages, Hkv, page_size, D)
+    src = xt.reshape(B, Hkv, max_pages, page_size, D).permute(0, 2, 1, 3, 4)
+    pool[torch.as_tensor(block_table.reshape(-1), dtype=torch.long)] = src.reshape(-1, Hkv, page_size, D)
+    return pool
+
+
+# ---------------------------------------------------------------------------
+# The five workloads.  Shapes follow the Qwen-family decoders of the paper's
+# experiments; budgets follow Sec. 5.2 (clamp) and App. B.1 (tau).
+# ---------------------------------------------------------------------------
+
+ADAPTIVE_5PCT = dict(mode=0, tau=0.1, r_lo_ppm=10_000, r_hi_ppm=50_000)
+ADAPTIVE_10PCT = dict(mode=0, tau=0.4, r_lo_ppm=50_000, r_hi_ppm=100_000)
+
+TINY = Recipe(
+    name="tiny-ref", layers=1, batch=1, heads=8, kv_heads=2, head_dim=64, dtype=FP32,
+    vis_len=576, vis_start=0, text_len=128, steps=16, planted_frac=0.05, seed=1,
+    beta_range=(1.0, 1.0), budget=ADAPTIVE_5PCT)
+
+QWEN7B = Recipe(
+    name="qwen2.5-vl-7b-decode", layers=28, batch=1, heads=28, kv_heads=4, head_dim=128,
+    dtype=BF16, vis_len=1296, vis_start=0, text_len=512 + 2048 + 1, steps=256,
+    planted_frac=0.03, seed=2, n_focus=4, focus_every=64, beta_range=(0.3, 0.85),
+    beta_sink=1.0, budget=ADAPTIVE_5PCT)
+
+
+def serving_recipe(seed=3, batch=32):
+    rng = _rng(seed, 0)
+    text = tuple(int(t) for t in rng.integers(512, 4097, size=batch))
+    seq_beta = tuple(float(x) for x in np.exp(rng.uniform(math.log(0.5), math.log(1.5), size=batch)))
+    return Recipe(
+        name="batched-serving-paged", layers=28, batch=batch, heads=28, kv_heads=4,
+        head_dim=128, dtype=BF16, vis_len=2304, vis_start=0, text_len=text, steps=64,
+        planted_frac=0.03, seed=seed, beta_range=(0.6, 1.0), seq_beta=seq_beta,
+        beta_sink=1.0, paged=True, page_size=16, budget=ADAPTIVE_5PCT)
+
+
+SERVING = serving_recipe()
+
+LONG = Recipe(
+    name="long-reasoning", layers=28, batch=8, heads=28, kv_heads=4, head_dim=128,
+    dtype=BF16, vis_len=4096, vis_start=0, text_len=16384, steps=512,
+    planted_frac=0.03, seed=4, beta_range=(0.3, 0.85), beta_sink=1.0, key_sigma=0.5,
+    budget=ADAPTIVE_5PCT)
+
+
+def sweep_recipe(vis_len: int, budget: dict, seed=5, batch=64):
+    return Recipe(
+        name=f"sweep-nv{vis_len}", layers=1, batch=batch, heads=32, kv_heads=8,
+        head_dim=128, dtype=BF16, vis_len=vis_len, vis_start=0, text_len=1024, steps=16,
+        planted_frac=0.03, seed=seed, beta_range=(0.3, 0.85), beta_sink=1.0, budget=budget)
+
+
+SWEEP_VIS = (576, 2304, 6400, 16384)
+SWEEP_BUDGETS = tuple(dict(mode=1, tau=0.1, ratio_ppm=r) for r in (10_000, 50_000, 200_000, 500_000)) \
+    + (ADAPTIVE_5PCT,)
+
+
+def shrink(r: Recipe, **kw) -> Recipe:
+    """A smaller copy of a recipe (tests)."""
+    return replace(r, **kw)
