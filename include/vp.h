@@ -1,0 +1,171 @@
+/*
+ * vp.h -- C ABI of libvp, a GB300 (sm_103a) implementation of one decode step
+ * of VisionPulse step-wise visual-pruned attention (arxiv 2605.31457).
+ *
+ * One call of vp_decode_step() runs, for every sequence of a batch and one
+ * attention layer acting as the anchor layer l_a (Sec. 4.2):
+ *   1. logits of the current query against every cached key      (Eq. 6's Z)
+ *   2. the temperature-scaled visual attention mass per head and
+ *      its head-max                                               (Eq. 5, Eq. 6, Sec. 4.3)
+ *   3. the step's retention budget K_t = M_vis,max * N_v, clamped  (Eq. 7, Sec. 5.2)
+ *   4. the top-K_t visual tokens by the head-averaged score S_i    (Eq. 2, Eq. 3)
+ *   5. attention over the kept visual tokens plus every text token (Sec. 4.2, Sec. 5.7)
+ *
+ * Conventions shared by every entry point:
+ *   - Tensors are caller-owned DEVICE memory unless stated otherwise; the
+ *     library never frees or retains them beyond the call.  The context owns
+ *     only its own workspace, allocated once in vp_init().
+ *   - vp_decode_step() allocates nothing, never synchronises the host and only
+ *     enqueues work on the caller's stream; its results are visible to later
+ *     work on that stream.
+ *   - Errors are returned as vp_status; nothing crosses the ABI as an
+ *     exception.  Invalid host-visible arguments are rejected before any work
+ *     is enqueued.  Per-sequence values that live on the device (spans, text
+ *     lengths, page ids) are checked by the kernels: an out-of-range value is
+ *     clamped or skipped, never dereferenced, and recorded in a device error
+ *     word that vp_check_errors() reports.
+ *   - A context serves one stream at a time; it is not thread-safe.
+ */
+#ifndef VP_H_
+#define VP_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  VP_OK = 0,
+  VP_ERR_INVALID_ARG = 1,     /* a host-visible argument is malformed          */
+  VP_ERR_UNSUPPORTED = 2,     /* valid, but a shape or mode this build lacks   */
+  VP_ERR_CAPACITY = 3,        /* batch or kept_cap exceeds what was configured */
+  VP_ERR_NOT_INITIALIZED = 4, /* NULL context                                  */
+  VP_ERR_CUDA = 5,            /* a CUDA runtime call failed (text in last_error)*/
+  VP_ERR_DEVICE_PRECOND = 6   /* vp_check_errors: a device-side check fired    */
+} vp_status;
+
+typedef enum { VP_BF16 = 0, VP_FP32 = 1 } vp_dtype;
+
+/* Budget modes (vp_budget.mode). */
+typedef enum {
+  VP_ADAPTIVE = 0,    /* K_t = ceil(M_vis,max(tau) * N_v) clamped to [K_lo, K_hi] (Eq. 7, Sec. 5.2) */
+  VP_FIXED_RATIO = 1, /* K_t = max(1, ceil(ratio * N_v))   (FastV-VP "Fix Ratio", Table 2)        */
+  VP_FIXED_K = 2,     /* K_t = min(fixed_k, N_v)           (Top-k budgeting, App. A.2)             */
+  VP_DENSE = 3        /* K_t = N_v: keep every visual token (full budget)                          */
+} vp_budget_mode;
+
+/* Static shapes, fixed for the life of a context (vp_init). */
+typedef struct {
+  int32_t max_batch;    /* largest batch a call may pass                          */
+  int32_t num_q_heads;  /* H, query heads of the layer                            */
+  int32_t num_kv_heads; /* Hkv, key/value heads; H % Hkv == 0, G = H / Hkv <= 16  */
+  int32_t head_dim;     /* D: 64 or 128                                           */
+  int32_t max_visual;   /* largest visual span N_v of any sequence (<= 32768)     */
+  int32_t max_seq;      /* largest live cache length N_v + text_len               */
+  vp_dtype dtype;       /* q, caches and out share this dtype                     */
+  int32_t paged;        /* 0: contiguous caches, 1: paged caches                  */
+  int32_t page_size;    /* tokens per page when paged (power of two, <= 256)      */
+} vp_config;
+
+/*
+ * One key or value cache.  Element (b, kv-head g, token t, dim d) lives at
+ *   contiguous: data + b*stride_b + g*stride_h + t*stride_t + d
+ *   paged:      data + page*stride_b + g*stride_h + (t % page_size)*stride_t + d,
+ *               page = block_table[b*max_pages + t / page_size]
+ * (strides in elements; the d axis is contiguous).  Every row (D elements)
+ * must start on a 16-byte boundary: data 16-byte aligned and every stride a
+ * multiple of 16 bytes.  A page id outside [0, num_pages) is skipped and
+ * flagged.
+ */
+typedef struct {
+  const void* data;
+  int64_t stride_b;            /* contiguous: sequence stride; paged: page stride  */
+  int64_t stride_h;            /* kv-head stride                                   */
+  int64_t stride_t;            /* token stride                                     */
+  const int32_t* block_table;  /* paged only: device [batch][max_pages]; else NULL */
+  int32_t max_pages;           /* paged only: row length of block_table            */
+  int32_t num_pages;           /* paged only: pages in the pool (bounds check)     */
+} vp_kv;
+
+/* Visual span of each sequence: tokens [vis_start[b], vis_start[b] + vis_len[b])
+ * of the live cache are visual (X_v of Sec. 4.2); all other live tokens are
+ * text (prompt, generated reasoning and the current token).  Device int32 [batch]. */
+typedef struct {
+  const int32_t* vis_start;
+  const int32_t* vis_len;
+} vp_span;
+
+typedef struct {
+  int32_t mode;        /* vp_budget_mode                                                 */
+  float tau;           /* Eq. 6 temperature for the mass, (0, 1]; 0.1 (5%) or 0.4 (10%)  */
+  float scale;         /* logit scale; 0 means 1/sqrt(D)                                 */
+  int32_t r_lo_ppm;    /* ADAPTIVE clamp, parts per million: K_lo = ceil(r_lo*N_v)       */
+  int32_t r_hi_ppm;    /*   K_hi = max(K_lo, floor(r_hi*N_v)); e.g. 10000 / 50000 (Sec. 5.2) */
+  int32_t ratio_ppm;   /* FIXED_RATIO ratio, parts per million                           */
+  int32_t fixed_k;     /* FIXED_K budget                                                 */
+  int32_t granularity; /* 0: one kept set per sequence, S averaged over all H heads (Eq. 2);
+                          1: one kept set per kv-head, S averaged over its G query heads  */
+} vp_budget;
+
+typedef struct vp_ctx vp_ctx;
+
+/* Creates a context for the given static shapes on the current CUDA device and
+ * allocates its workspace (logit scratch, split partials, counters) once.
+ * Returns VP_ERR_INVALID_ARG / VP_ERR_UNSUPPORTED for bad shapes, VP_ERR_CUDA
+ * when allocation fails.  *out_ctx is NULL on failure. */
+vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx);
+
+/*
+ * One VisionPulse decode step (Sec. 4.2-4.3) for `batch` sequences.
+ *   q            [batch][H][D] cfg.dtype, query of the current token (post-RoPE).
+ *   k_cache,
+ *   v_cache      caches holding N_v + text_len[b] live tokens of sequence b,
+ *                the current token already appended (it counts in text_len).
+ *   visual_span  device spans; 0 <= vis_start <= text_len, vis_len <= max_visual.
+ *   text_len     device int32 [batch], >= 1; N_v + text_len <= max_seq.
+ *   budget       host struct, see vp_budget.
+ *   out          [batch][H][D] cfg.dtype: softmax attention of q over the kept
+ *                visual tokens plus all text tokens (dropped tokens are
+ *                excluded from the normaliser).
+ *   kept_idx     int32 [batch][kept_cap] (granularity 1: [batch][Hkv][kept_cap]):
+ *                kept visual indices, relative to vis_start, ascending; the
+ *                K_t largest S_i, ties to the lower index; unused slots = -1.
+ *   kept_cap     must be >= the largest K_t the budget can produce for
+ *                max_visual tokens, else VP_ERR_CAPACITY (nothing enqueued).
+ *   kept_count   int32 [batch] (granularity 1: [batch][Hkv]): K_t.
+ *   mass         float [batch][H]: m_{t,h} of Eq. 5 under the Eq. 6 temperature.
+ *   mass_stats   float [batch][4] or NULL: { M_vis(tau), M_vis,max(tau),
+ *                M_vis(tau = 1), (float)K_t }.
+ *   cuda_stream  cudaStream_t to enqueue on (NULL = legacy default stream).
+ */
+vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
+                         const vp_kv* k_cache, const vp_kv* v_cache,
+                         const vp_span* visual_span, const int32_t* text_len,
+                         const vp_budget* budget, void* out,
+                         int32_t* kept_idx, int32_t kept_cap, int32_t* kept_count,
+                         float* mass, float* mass_stats, void* cuda_stream);
+
+/* Largest K_t the budget can produce for n_visual tokens (the kept_cap a
+ * caller must provide); -1 for an invalid budget.  Host only, no CUDA. */
+int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual);
+
+/* Text of the last error on this context ("" if none).  Valid until the next
+ * call on the context.  Accepts NULL (returns the text of the last vp_init
+ * failure in this thread). */
+const char* vp_last_error(const vp_ctx* ctx);
+
+/* Synchronises `cuda_stream`, then reads and clears the device error word.
+ * Returns VP_OK, VP_ERR_DEVICE_PRECOND (with the failed checks in
+ * vp_last_error) or VP_ERR_CUDA. */
+vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream);
+
+/* Releases the workspace and the context; NULL is a no-op.  Waits for the
+ * device to finish work that may still use the workspace. */
+void vp_free(vp_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VP_H_ */

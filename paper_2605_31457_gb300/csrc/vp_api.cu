@@ -1,0 +1,307 @@
+// Host side of libvp: argument checking, workspace ownership, launch planning
+// and the extern "C" entry points declared in include/vp.h.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+
+#include "vp.h"
+#include "vp_internal.h"
+
+struct vp_ctx {
+  vp_config cfg;
+  int device = 0;
+  int num_sms = 0;
+  int ns_max = 1, nk_max = 1;
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  float* z_ws = nullptr;
+  float* split_st = nullptr;
+  float* split_o = nullptr;
+  float* gpart_o = nullptr;
+  float* gpart_st = nullptr;
+  unsigned* tickets = nullptr;
+  unsigned* err = nullptr;
+  std::string last_error;
+};
+
+namespace {
+
+thread_local std::string g_init_error;
+
+constexpr int64_t kPpm = 1000000;
+constexpr int kMaxVisual = 32768;  // score keys of one sequence fit in shared memory
+constexpr int kMaxHeads = 128;
+constexpr int kMaxGroup = 16;
+
+vp_status fail(vp_ctx* ctx, vp_status st, const std::string& msg) {
+  if (ctx) ctx->last_error = msg;
+  else g_init_error = msg;
+  return st;
+}
+
+vp_status cuda_fail(vp_ctx* ctx, const char* what, cudaError_t e) {
+  return fail(ctx, VP_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Largest K_t the budget yields for n visual tokens (K_t is non-decreasing in
+// N_v in every mode, so the bound for max_visual covers every sequence).
+int32_t max_kept(const vp_budget& bd, int32_t n) {
+  if (n <= 0) return 0;
+  switch (bd.mode) {
+    case VP_DENSE: return n;
+    case VP_FIXED_K: return bd.fixed_k < n ? (bd.fixed_k < 0 ? 0 : bd.fixed_k) : n;
+    case VP_FIXED_RATIO: {
+      int64_t k = ceil_div((int64_t)bd.ratio_ppm * n, kPpm);
+      if (k < 1) k = 1;
+      return (int32_t)(k < n ? k : n);
+    }
+    case VP_ADAPTIVE: {
+      const int64_t k_lo = ceil_div((int64_t)bd.r_lo_ppm * n, kPpm);
+      int64_t k_hi = (int64_t)bd.r_hi_ppm * n / kPpm;
+      if (k_hi < k_lo) k_hi = k_lo;
+      return (int32_t)(k_hi < n ? k_hi : n);
+    }
+    default: return -1;
+  }
+}
+
+bool budget_ok(const vp_budget& bd, std::string* why) {
+  if (bd.mode < VP_ADAPTIVE || bd.mode > VP_DENSE) { *why = "budget.mode out of range"; return false; }
+  if (!(bd.tau > 0.f) || !isfinite(bd.tau)) { *why = "budget.tau must be finite and > 0"; return false; }
+  if (!(bd.scale >= 0.f) || !isfinite(bd.scale)) { *why = "budget.scale must be finite and >= 0"; return false; }
+  if (bd.r_lo_ppm < 0 || bd.r_lo_ppm > kPpm || bd.r_hi_ppm < 0 || bd.r_hi_ppm > kPpm) {
+    *why = "budget clamp ratios must lie in [0, 1000000] ppm"; return false;
+  }
+  if (bd.ratio_ppm < 0 || bd.ratio_ppm > kPpm) { *why = "budget.ratio_ppm must lie in [0, 1000000]"; return false; }
+  if (bd.fixed_k < 0) { *why = "budget.fixed_k must be >= 0"; return false; }
+  if (bd.granularity != 0 && bd.granularity != 1) { *why = "budget.granularity must be 0 or 1"; return false; }
+  return true;
+}
+
+bool kv_ok(const vp_ctx* ctx, const vp_kv* kv, const char* name, std::string* why) {
+  const size_t esz = ctx->cfg.dtype == VP_BF16 ? 2 : 4;
+  char buf[160];
+  if (!kv || !kv->data) { snprintf(buf, sizeof buf, "%s: NULL cache", name); *why = buf; return false; }
+  if (!aligned16(kv->data)) { snprintf(buf, sizeof buf, "%s: data must be 16-byte aligned", name); *why = buf; return false; }
+  const int64_t strides[3] = {kv->stride_b, kv->stride_h, kv->stride_t};
+  for (int64_t s : strides) {
+    if (s < 0 || ((uint64_t)s * esz) % 16 != 0) {
+      snprintf(buf, sizeof buf, "%s: strides must be >= 0 and multiples of 16 bytes", name); *why = buf; return false;
+    }
+  }
+  if (ctx->cfg.paged) {
+    if (!kv->block_table || kv->max_pages < 1 || kv->num_pages < 1) {
+      snprintf(buf, sizeof buf, "%s: paged cache needs block_table, max_pages >= 1, num_pages >= 1", name);
+      *why = buf; return false;
+    }
+  } else if (kv->block_table) {
+    snprintf(buf, sizeof buf, "%s: block_table given but the context is not paged", name); *why = buf; return false;
+  }
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual) {
+  if (!budget || n_visual < 0) return -1;
+  std::string why;
+  if (!budget_ok(*budget, &why)) return -1;
+  return max_kept(*budget, n_visual);
+}
+
+vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx) {
+  if (!out_ctx) return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: out_ctx is NULL");
+  *out_ctx = nullptr;
+  if (!cfg) return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: cfg is NULL");
+  const vp_config& c = *cfg;
+  if (c.max_batch < 1 || c.num_q_heads < 1 || c.num_kv_heads < 1)
+    return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: max_batch, num_q_heads and num_kv_heads must be >= 1");
+  if (c.num_q_heads % c.num_kv_heads != 0)
+    return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: num_q_heads must be a multiple of num_kv_heads");
+  if (c.dtype != VP_BF16 && c.dtype != VP_FP32)
+    return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: dtype must be VP_BF16 or VP_FP32");
+  if (c.max_visual < 0 || c.max_seq < c.max_visual + 1)
+    return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: need 0 <= max_visual and max_seq >= max_visual + 1");
+  if (c.paged != 0 && c.paged != 1) return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: paged must be 0 or 1");
+  if (c.paged && (c.page_size < 1 || c.page_size > 256 || (c.page_size & (c.page_size - 1))))
+    return fail(nullptr, VP_ERR_INVALID_ARG, "vp_init: page_size must be a power of two in [1, 256]");
+  if (c.head_dim != 64 && c.head_dim != 128)
+    return fail(nullptr, VP_ERR_UNSUPPORTED, "vp_init: head_dim must be 64 or 128");
+  if (c.num_q_heads / c.num_kv_heads > kMaxGroup || c.num_q_heads > kMaxHeads)
+    return fail(nullptr, VP_ERR_UNSUPPORTED, "vp_init: needs G = H / Hkv <= 16 and H <= 128");
+  if (c.max_visual > kMaxVisual)
+    return fail(nullptr, VP_ERR_UNSUPPORTED, "vp_init: max_visual above 32768 is not supported");
+
+  vp_ctx* ctx = new vp_ctx();
+  ctx->cfg = c;
+  cudaError_t e = cudaGetDevice(&ctx->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, ctx->device);
+  if (e != cudaSuccess) {
+    vp_status st = cuda_fail(nullptr, "vp_init: no usable CUDA device", e);
+    delete ctx;
+    return st;
+  }
+  const int H = c.num_q_heads, Hkv = c.num_kv_heads, G = H / Hkv, D = c.head_dim;
+  // Split counts: enough CTAs for a batch of one sequence to cover every SM
+  // four times, and at least 32 work units (tokens) per split.
+  const int64_t work_max = (int64_t)c.max_visual + 2LL * c.max_seq;
+  ctx->ns_max = (int)std::max<int64_t>(1, std::min<int64_t>({256, ceil_div(4LL * ctx->num_sms, Hkv), ceil_div(work_max, 32)}));
+  ctx->nk_max = (int)std::max<int64_t>(1, std::min<int64_t>(64, ceil_div(2LL * ctx->num_sms, Hkv)));
+
+  const size_t B = (size_t)c.max_batch;
+  const size_t sz_z = B * H * (size_t)std::max(c.max_visual, 1) * 4;
+  const size_t sz_st = B * H * (size_t)ctx->ns_max * vp::ST_N * 4;
+  const size_t sz_o = B * H * (size_t)ctx->ns_max * D * 4;
+  const size_t sz_go = B * Hkv * (size_t)ctx->nk_max * G * D * 4;
+  const size_t sz_gs = B * Hkv * (size_t)ctx->nk_max * G * 2 * 4;
+  const size_t sz_t = B * Hkv * 4;
+  size_t off = 0;
+  const size_t o_z = off; off = round_up(off + sz_z, 256);
+  const size_t o_st = off; off = round_up(off + sz_st, 256);
+  const size_t o_o = off; off = round_up(off + sz_o, 256);
+  const size_t o_go = off; off = round_up(off + sz_go, 256);
+  const size_t o_gs = off; off = round_up(off + sz_gs, 256);
+  const size_t o_t = off; off = round_up(off + sz_t, 256);
+  const size_t o_e = off; off = round_up(off + 4, 256);
+  ctx->ws_bytes = off;
+  e = cudaMalloc(&ctx->ws, ctx->ws_bytes);
+  if (e != cudaSuccess) {
+    vp_status st = cuda_fail(nullptr, "vp_init: workspace allocation failed", e);
+    delete ctx;
+    return st;
+  }
+  char* base = static_cast<char*>(ctx->ws);
+  ctx->z_ws = reinterpret_cast<float*>(base + o_z);
+  ctx->split_st = reinterpret_cast<float*>(base + o_st);
+  ctx->split_o = reinterpret_cast<float*>(base + o_o);
+  ctx->gpart_o = reinterpret_cast<float*>(base + o_go);
+  ctx->gpart_st = reinterpret_cast<float*>(base + o_gs);
+  ctx->tickets = reinterpret_cast<unsigned*>(base + o_t);
+  ctx->err = reinterpret_cast<unsigned*>(base + o_e);
+  e = cudaMemset(ctx->ws, 0, ctx->ws_bytes);
+  if (e == cudaSuccess) e = vp::configure_kernels(c.max_visual);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    vp_status st = cuda_fail(nullptr, "vp_init: workspace set-up failed", e);
+    cudaFree(ctx->ws);
+    delete ctx;
+    return st;
+  }
+  *out_ctx = ctx;
+  return VP_OK;
+}
+
+vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
+                         const vp_kv* k_cache, const vp_kv* v_cache,
+                         const vp_span* visual_span, const int32_t* text_len,
+                         const vp_budget* budget, void* out,
+                         int32_t* kept_idx, int32_t kept_cap, int32_t* kept_count,
+                         float* mass, float* mass_stats, void* cuda_stream) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  ctx->last_error.clear();
+  const vp_config& c = ctx->cfg;
+  if (batch < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: batch < 0");
+  if (batch > c.max_batch) return fail(ctx, VP_ERR_CAPACITY, "vp_decode_step: batch exceeds max_batch");
+  if (!budget) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: budget is NULL");
+  std::string why;
+  if (!budget_ok(*budget, &why)) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: " + why);
+  const int32_t need = max_kept(*budget, c.max_visual);
+  if (kept_cap < 0 || kept_cap < need) {
+    return fail(ctx, VP_ERR_CAPACITY, "vp_decode_step: kept_cap " + std::to_string(kept_cap) +
+                " is below the largest budget " + std::to_string(need));
+  }
+  if (batch == 0) return VP_OK;
+  if (!q || !out || !text_len || !visual_span || !visual_span->vis_start || !visual_span->vis_len ||
+      !kept_count || !mass || (kept_cap > 0 && !kept_idx))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: NULL tensor argument");
+  if (!aligned16(q) || !aligned16(out)) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: q and out must be 16-byte aligned");
+  if (!kv_ok(ctx, k_cache, "k_cache", &why) || !kv_ok(ctx, v_cache, "v_cache", &why))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_step: " + why);
+
+  const int H = c.num_q_heads, Hkv = c.num_kv_heads;
+  vp::StepParams p;
+  memset(&p, 0, sizeof p);
+  p.dtype = c.dtype;
+  p.B = batch; p.H = H; p.Hkv = Hkv; p.G = H / Hkv; p.D = c.head_dim;
+  p.max_visual = c.max_visual; p.max_seq = c.max_seq;
+  p.paged = c.paged; p.page_size = c.paged ? c.page_size : 1;
+  p.page_shift = 0;
+  while ((1 << p.page_shift) < p.page_size) ++p.page_shift;
+  p.q = q;
+  p.k = vp::KvView{k_cache->data, k_cache->stride_b, k_cache->stride_h, k_cache->stride_t,
+                   k_cache->block_table, k_cache->max_pages, k_cache->num_pages};
+  p.v = vp::KvView{v_cache->data, v_cache->stride_b, v_cache->stride_h, v_cache->stride_t,
+                   v_cache->block_table, v_cache->max_pages, v_cache->num_pages};
+  p.vis_start = visual_span->vis_start;
+  p.vis_len = visual_span->vis_len;
+  p.text_len = text_len;
+  p.mode = budget->mode;
+  p.granularity = budget->granularity;
+  p.inv_tau = 1.0f / budget->tau;
+  const float scale = budget->scale > 0.f ? budget->scale : 1.0f / sqrtf((float)c.head_dim);
+  p.c_log2 = scale * 1.4426950408889634f;
+  p.r_lo_ppm = budget->r_lo_ppm; p.r_hi_ppm = budget->r_hi_ppm;
+  p.ratio_ppm = budget->ratio_ppm; p.fixed_k = budget->fixed_k;
+  p.out = out; p.kept_idx = kept_idx; p.kept_cap = kept_cap; p.kept_count = kept_count;
+  p.mass = mass; p.mass_stats = mass_stats;
+  p.z_ws = ctx->z_ws; p.split_st = ctx->split_st; p.split_o = ctx->split_o;
+  p.gpart_o = ctx->gpart_o; p.gpart_st = ctx->gpart_st; p.tickets = ctx->tickets; p.err = ctx->err;
+  p.ns_max = ctx->ns_max; p.nk_max = ctx->nk_max;
+  const int64_t units = (int64_t)batch * Hkv;
+  p.ns = (int)std::max<int64_t>(1, std::min<int64_t>(ctx->ns_max, ceil_div(4LL * ctx->num_sms, units)));
+  p.nk = (int)std::max<int64_t>(1, std::min<int64_t>({(int64_t)ctx->nk_max, ceil_div(2LL * ctx->num_sms, units),
+                                                       std::max<int64_t>(1, ceil_div(kept_cap, 16))}));
+
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = vp::launch_score(p, st);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: score kernel launch", e);
+  e = vp::launch_select(p, st);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: select kernel launch", e);
+  e = vp::launch_gather(p, st);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: gather kernel launch", e);
+  return VP_OK;
+}
+
+const char* vp_last_error(const vp_ctx* ctx) {
+  return ctx ? ctx->last_error.c_str() : g_init_error.c_str();
+}
+
+vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = cudaStreamSynchronize(st);
+  unsigned word = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&word, ctx->err, sizeof word, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && word) e = cudaMemset(ctx->err, 0, sizeof word);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_check_errors", e);
+  if (!word) { ctx->last_error.clear(); return VP_OK; }
+  std::string msg = "device checks failed:";
+  if (word & vp::ERR_SPAN) msg += " visual span outside the live cache or above max_visual;";
+  if (word & vp::ERR_TEXT) msg += " text_len < 1;";
+  if (word & vp::ERR_LEN) msg += " vis_len + text_len above max_seq;";
+  if (word & vp::ERR_PAGE) msg += " block table entry outside the pool;";
+  if (word & vp::ERR_KEPT) msg += " kept index outside the visual span;";
+  if (word & vp::ERR_NONFINITE) msg += " non-finite importance score;";
+  return fail(ctx, VP_ERR_DEVICE_PRECOND, msg);
+}
+
+void vp_free(vp_ctx* ctx) {
+  if (!ctx) return;
+  if (ctx->ws) cudaFree(ctx->ws);
+  delete ctx;
+}
+
+}  // extern "C"

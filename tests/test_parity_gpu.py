@@ -1,0 +1,222 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Small cases span several 32-token groups, split boundaries and ragged tails;
+the full-size cases run the launch configuration the benchmark times and
+compare every (or a sample of) sequence with the oracle.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import vp_oracle as O
+from paper_2605_31457_gb300 import workloads as W
+
+from . import vp_harness as Hn
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def vp(lib):
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    return lib
+
+
+def small(**kw):
+    base = dict(name="small", layers=1, batch=3, heads=28, kv_heads=4, head_dim=128, dtype=W.BF16,
+                vis_len=(300, 577, 64), vis_start=(0, 13, 40), text_len=(517, 70, 129), steps=1,
+                planted_frac=0.04, seed=11, beta_range=(0.3, 0.9), beta_sink=1.0,
+                budget=W.ADAPTIVE_5PCT)
+    base.update(kw)
+    return W.Recipe(**base)
+
+
+# ------------------------------------------------------------------ tiny ref
+
+def test_tiny_reference_all_steps(vp):
+    """The 16-step fp32 reference workload, every step against the oracle."""
+    r = W.TINY
+    li = W.make_layer(r, 0, t_cap=r.capacity())
+    qs = W.make_queries(r, 0, li)
+    rep = {}
+    for step in range(r.steps):
+        inp = Hn.make_inputs(r, 0, step, t_cap=r.capacity(), q_override=qs[step])
+        Hn.check_all(vp, inp, r.budget, report=rep)
+    assert rep.get("max_out_err", 0) < 1e-5
+
+
+# --------------------------------------------------------- shapes and modes
+
+@pytest.mark.parametrize("dtype,D", [(W.BF16, 128), (W.BF16, 64), (W.FP32, 128), (W.FP32, 64)])
+def test_dtypes_and_head_dims(vp, dtype, D):
+    r = small(dtype=dtype, head_dim=D)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget)
+
+
+@pytest.mark.parametrize("H,Hkv", [(8, 8), (16, 1), (32, 8), (12, 4), (28, 4)])
+def test_group_sizes(vp, H, Hkv):
+    r = small(heads=H, kv_heads=Hkv)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget)
+
+
+@pytest.mark.parametrize("budget", [
+    dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=10_000),
+    dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=50_000),
+    dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000),
+    dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000),
+    dict(mode=O.FIXED_K, tau=0.1, fixed_k=256),
+    dict(mode=O.DENSE, tau=0.1),
+    W.ADAPTIVE_10PCT,
+    dict(mode=O.ADAPTIVE, tau=0.4, r_lo_ppm=0, r_hi_ppm=1_000_000),
+    dict(mode=O.ADAPTIVE, tau=1.0, r_lo_ppm=0, r_hi_ppm=1_000_000),
+])
+def test_budget_modes(vp, budget):
+    r = small()
+    Hn.check_all(vp, Hn.make_inputs(r), budget)
+
+
+@pytest.mark.parametrize("budget", [dict(W.ADAPTIVE_5PCT, granularity=1),
+                                    dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000, granularity=1)])
+def test_per_kv_head_selection(vp, budget):
+    r = small()
+    Hn.check_all(vp, Hn.make_inputs(r), budget)
+
+
+def test_paged_cache(vp):
+    r = small(batch=4, vis_len=(300, 577, 64, 1000), vis_start=(0, 13, 40, 0),
+              text_len=(517, 70, 129, 33), paged=True, page_size=16)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget)
+
+
+def test_paged_cache_other_page_size(vp):
+    r = small(paged=True, page_size=64, dtype=W.FP32, head_dim=64, heads=8, kv_heads=2)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget)
+
+
+def test_explicit_logit_scale(vp):
+    r = small()
+    Hn.check_all(vp, Hn.make_inputs(r), dict(r.budget, scale=0.05))
+
+
+# ---------------------------------------------------------------- edge cases
+
+def test_edge_lengths(vp):
+    """Empty visual span, one visual token, only the current text token,
+    and a visual span starting after the whole prompt."""
+    r = small(batch=5, vis_len=(0, 1, 33, 700, 16), vis_start=(0, 0, 1, 0, 9),
+              text_len=(5, 1, 1, 1, 9))
+    for budget in (r.budget, dict(mode=O.DENSE, tau=0.1), dict(mode=O.FIXED_K, tau=0.1, fixed_k=3)):
+        Hn.check_all(vp, Hn.make_inputs(r), budget)
+
+
+def test_zero_query_ties_go_to_lower_indices(vp):
+    r = small()
+    q = np.zeros((r.batch, r.heads, r.head_dim), dtype=np.float32)
+    inp = Hn.make_inputs(r, q_override=q)
+    gpu = Hn.check_all(vp, inp, dict(mode=O.FIXED_K, tau=0.1, fixed_k=17))
+    for b in range(r.batch):
+        k = int(gpu["count"][b][0])
+        np.testing.assert_array_equal(gpu["kept"][b][0][:k], np.arange(k))
+
+
+def test_planted_keys_recovered_on_gpu(vp):
+    r = small(beta_range=(1.2, 1.2), beta_sink=0.0, planted_frac=0.03)
+    inp = Hn.make_inputs(r)
+    li = W.make_layer(r, 0, t_cap=r.capacity(1))
+    budget = dict(mode=O.FIXED_K, tau=0.1, fixed_k=64)
+    gpu = Hn.check_all(vp, inp, budget)
+    for b in range(r.batch):
+        planted = set(li.planted[0][b].tolist())
+        kept = set(gpu["kept"][b][0][: int(gpu["count"][b][0])].tolist())
+        assert planted <= kept
+
+
+def test_batch_below_max_batch_and_repeat_calls(vp):
+    """A context sized for more sequences, called twice: same results."""
+    r = small()
+    inp = Hn.make_inputs(r)
+    dev = Hn.Device(vp, inp, r.budget, max_batch=8, max_seq=4096)
+    try:
+        a = dev.run()
+        b = dev.run()
+    finally:
+        dev.close()
+    for key in a:
+        np.testing.assert_array_equal(a[key], b[key])
+    for s in range(r.batch):
+        Hn.compare_seq(inp, a, s, r.budget)
+
+
+def test_device_precondition_is_reported_not_faulted(vp):
+    """A visual span past the live cache is clamped and reported."""
+    r = small(batch=1, vis_len=(64,), vis_start=(0,), text_len=(32,))
+    inp = Hn.make_inputs(r)
+    dev = Hn.Device(vp, inp, r.budget)
+    try:
+        dev.vs.fill_(50)          # vis_start > text_len
+        dev.run(check_errors=False)
+        st = vp.vp_check_errors(dev.ctx, check=False)
+        assert st == vp.VP_ERR_DEVICE_PRECOND
+        assert "visual span" in vp.vp_last_error(dev.ctx)
+        assert vp.vp_check_errors(dev.ctx, check=False) == vp.VP_OK   # cleared
+    finally:
+        dev.close()
+
+
+def test_capacity_and_argument_errors(vp):
+    r = small(batch=1, vis_len=(64,), vis_start=(0,), text_len=(32,))
+    inp = Hn.make_inputs(r)
+    dev = Hn.Device(vp, inp, r.budget)
+    try:
+        st = vp.vp_decode_step(dev.ctx, 1, dev.q, dev.kc, dev.vc, dev.span, dev.tl, dev.budget, dev.out,
+                               dev.kept, 1, dev.count, dev.mass, dev.stats, check=False)
+        assert st == vp.VP_ERR_CAPACITY
+        st = vp.vp_decode_step(dev.ctx, 2, dev.q, dev.kc, dev.vc, dev.span, dev.tl, dev.budget, dev.out,
+                               dev.kept, dev.kept_cap, dev.count, dev.mass, dev.stats, check=False)
+        assert st == vp.VP_ERR_CAPACITY
+        bad = vp.make_budget(tau=-1.0)
+        st = vp.vp_decode_step(dev.ctx, 1, dev.q, dev.kc, dev.vc, dev.span, dev.tl, bad, dev.out,
+                               dev.kept, dev.kept_cap, dev.count, dev.mass, dev.stats, check=False)
+        assert st == vp.VP_ERR_INVALID_ARG
+        odd = vp.vp_kv(dev.k_t.data_ptr() + 2, dev.kc.stride_b, dev.kc.stride_h, dev.kc.stride_t, None, 0, 0)
+        st = vp.vp_decode_step(dev.ctx, 1, dev.q, odd, dev.vc, dev.span, dev.tl, dev.budget, dev.out,
+                               dev.kept, dev.kept_cap, dev.count, dev.mass, dev.stats, check=False)
+        assert st == vp.VP_ERR_INVALID_ARG
+        assert vp.vp_check_errors(dev.ctx, check=False) == vp.VP_OK
+    finally:
+        dev.close()
+
+
+# -------------------------------------------------------------- full sizes
+
+def test_qwen7b_full_size_layer(vp):
+    """The benchmarked workload (B = 1, 28/4 heads, 1296 visual + 2561 text,
+    bf16) at two decode steps of one layer: every output against the oracle."""
+    r = W.QWEN7B
+    t_cap = r.capacity(64)
+    li = W.make_layer(r, 3, t_cap=t_cap)
+    qs = W.make_queries(r, 3, li, steps=64)
+    rep = {}
+    for step in (0, 63):
+        inp = Hn.make_inputs(r, 3, step, t_cap=t_cap, q_override=qs[step])
+        Hn.check_all(vp, inp, r.budget, report=rep)
+        Hn.check_all(vp, inp, W.ADAPTIVE_10PCT, report=rep)
+
+
+def test_serving_paged_full_size_layer(vp):
+    """Batched serving: B = 32, paged (page 16), 2304 visual, text 512..4096."""
+    r = W.SERVING
+    inp = Hn.make_inputs(r, 0, 0)
+    gpu = Hn.check_all(vp, inp, r.budget, seqs=range(0, 32, 3))
+    assert len(set(gpu["count"][:, 0].tolist())) > 1, "budgets should differ across the batch"
+
+
+@pytest.mark.parametrize("nv", [576, 2304])
+def test_sweep_points(vp, nv):
+    for budget in W.SWEEP_BUDGETS:
+        r = W.sweep_recipe(nv, budget)
+        Hn.check_all(vp, Hn.make_inputs(r), budget, seqs=(0, 31, 63))
