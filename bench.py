@@ -1,0 +1,466 @@
+#!/usr/bin/env python3
+"""Benchmark of the VisionPulse pruned decode step on GB300.
+
+Workload (default): a Qwen2.5-VL-7B-shaped decoder, 28 layers of 28 query /
+4 kv heads, head_dim 128, bf16 caches, batch 1, 1296 visual + 2561 text
+tokens (512 prompt + 2048 generated + the current token) at the first step,
+one text token appended per step.  A step is one vp_decode_step call per
+layer (28 calls, each layer acting as its own anchor layer), i.e. the whole
+five-stage hot path over every layer.
+
+Prints one JSON line (rank 0).  `value` is decode steps per second with the
+caches resident in HBM (per-step CUDA graphs of the 28 calls, timed with CUDA
+events); `e2e` is the same metric through the C ABI with the step's query and
+appended K/V copied in from pinned host memory and the results copied back.
+`--impl reference` times the CPU oracle instead (rank 0, host cores).
+"""
+
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "pruned decode-attention steps/sec and achieved HBM GB/s (% of GB300 peak) on 1 GPU"
+UNIT = "steps/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU-baseline leg")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
+    return ap.parse_args(argv)
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# --------------------------------------------------------------- algorithmic bytes
+
+def call_bytes(r, n_visual, text_len, kept):
+    """Algorithmic HBM bytes of one layer call for one sequence, split by kernel:
+    score reads all visual K, text K and V and q; gather reads the kept visual
+    V rows and writes out."""
+    esz = 2 if r.dtype == "bf16" else 4
+    row = r.kv_heads * r.head_dim * esz
+    qo = r.heads * r.head_dim * esz
+    score = n_visual * row + 2 * text_len * row + qo
+    gather = kept * row + qo
+    return score, gather
+
+
+# ------------------------------------------------------------------ clock sampling
+
+class ClockSampler:
+    """Samples the SM clock and the clock-event (throttle) reasons through NVML
+    in a background thread while the timed region runs."""
+
+    REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+               0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+               0x100: "display_clock_setting"}
+
+    def __init__(self, torch_device, interval=0.002):
+        self.interval = interval
+        self.samples = []
+        self.err = None
+        self.h = None
+        try:
+            self.nvml = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.nvml.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit failed")
+            import torch
+            p = torch.cuda.get_device_properties(torch_device)
+            bus = f"{getattr(p, 'pci_domain_id', 0):08x}:{p.pci_bus_id:02x}:{p.pci_device_id:02x}.0".encode()
+            h = ctypes.c_void_p()
+            if self.nvml.nvmlDeviceGetHandleByPciBusId_v2(ctypes.c_char_p(bus), ctypes.byref(h)) != 0:
+                if self.nvml.nvmlDeviceGetHandleByIndex_v2(0, ctypes.byref(h)) != 0:
+                    raise OSError("no NVML handle")
+            self.h = h
+            mx = ctypes.c_uint(0)
+            self.nvml.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx))
+            self.max_mhz = mx.value
+            fn = getattr(self.nvml, "nvmlDeviceGetCurrentClocksEventReasons", None)
+            self.reasons_fn = fn or self.nvml.nvmlDeviceGetCurrentClocksThrottleReasons
+        except Exception as e:  # NVML is optional: report why clocks are missing
+            self.err = str(e)
+        self._stop = threading.Event()
+        self._t = None
+
+    def _loop(self):
+        clk = ctypes.c_uint(0)
+        rs = ctypes.c_ulonglong(0)
+        while not self._stop.is_set():
+            if self.nvml.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(clk)) == 0 and \
+                    self.reasons_fn(self.h, ctypes.byref(rs)) == 0:
+                self.samples.append((clk.value, rs.value))
+            time.sleep(self.interval)
+
+    def start(self):
+        if self.h is not None:
+            self._t = threading.Thread(target=self._loop, daemon=True)
+            self._t.start()
+
+    def stop(self):
+        if self._t is None:
+            return {"error": self.err or "NVML unavailable"}
+        self._stop.set()
+        self._t.join()
+        busy = [s for s in self.samples if not (s[1] & 0x1)] or self.samples
+        seen = 0
+        for _, r in busy:
+            seen |= r
+        names = [n for bit, n in self.REASONS.items() if seen & bit and bit != 0x1]
+        return {"sm_mhz": statistics.median(c for c, _ in busy) if busy else None,
+                "sm_max_mhz": self.max_mhz, "reasons": names, "samples": len(busy),
+                "source": "NVML, 2 ms sampling during the timed region"}
+
+
+# --------------------------------------------------------------------- oracle legs
+
+def _oracle_worker(args):
+    """Runs in a spawned process with single-threaded BLAS: times the oracle
+    on a sample of layer calls; returns seconds per layer call."""
+    recipe_name, layers, steps0, budget_s, max_calls = args
+    from paper_2605_31457_gb300 import workloads as W
+    from oracle import vp_oracle as O
+    r = getattr(W, recipe_name)
+    t_cap = r.capacity(steps0 + max_calls + 1)
+    times = []
+    cache = {}
+    t_start = time.perf_counter()
+    for n in range(max_calls):
+        layer = layers[n % len(layers)]
+        if layer not in cache:
+            li = W.make_layer(r, layer, t_cap=t_cap)
+            q = W.make_queries(r, layer, li, steps=steps0 + max_calls + 1)
+            cache[layer] = (W.round_to(li.k, r.dtype).double().numpy(),
+                            W.round_to(li.v, r.dtype).double().numpy(),
+                            W.round_to(q, r.dtype).double().numpy())
+        k, v, q = cache[layer]
+        s = steps0 + n
+        t0 = time.perf_counter()
+        for b in range(r.batch):
+            O.decode_step(q[s, b], k[b], v[b], int(r.vis_starts[b]), int(r.vis_lens[b]),
+                          int(r.text_lens[b]) + s, **r.budget)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() - t_start > budget_s:
+            break
+    return times
+
+
+def oracle_times(recipe_name, layers, steps0, budget_s, max_calls):
+    env_keys = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+    old = {k: os.environ.get(k) for k in env_keys}
+    for k in env_keys:
+        os.environ[k] = "1"
+    try:
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(1) as pool:
+            return pool.apply(_oracle_worker, ((recipe_name, layers, steps0, budget_s, max_calls),))
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    from paper_2605_31457_gb300 import workloads as W
+    r = W.QWEN7B
+    n = args.warmup + args.steps
+    times = oracle_times("QWEN7B", list(range(4)), 0, budget_s=1e9, max_calls=n)
+    timed = times[args.warmup:]
+    per_call = sum(timed) / len(timed)
+    ms_step = per_call * r.layers * 1e3
+    value = 1e3 / ms_step
+    sample = (f"each step = 1 of the {r.layers} layer calls of a decode step (layers 0-3 in turn), "
+              f"scaled x{r.layers} to a full step; {len(timed)} timed calls")
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(r),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(r):
+    return {"workload": (f"{r.name}: {r.layers} layers x {r.heads} q / {r.kv_heads} kv heads, "
+                         f"head_dim {r.head_dim}, {r.dtype}, batch {r.batch}, "
+                         f"{int(r.vis_lens[0])} visual + {int(r.text_lens[0])} text tokens at step 0 "
+                         f"(+1 text token per step), budget tau={r.budget['tau']} clamp "
+                         f"[{r.budget['r_lo_ppm'] / 1e4:g}%, {r.budget['r_hi_ppm'] / 1e4:g}%]"),
+            "global_batch": r.batch, "layers": r.layers,
+            "l2": "no flush: each step streams ~0.18 GB of K/V over 28 layers, above the 129 MB L2"}
+
+
+# ------------------------------------------------------------------------ our arm
+
+def run_ours(args, rank, world, local):
+    import numpy as np
+    import torch
+    from paper_2605_31457_gb300 import build as _build
+    _build.ensure_built()
+    from paper_2605_31457_gb300 import vp, workloads as W
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    r = W.QWEN7B
+    L, B, H, Hkv, D = r.layers, r.batch, r.heads, r.kv_heads, r.head_dim
+    S = args.warmup + args.steps
+    t_cap = r.capacity(S + 1)
+    nv0, tl0 = int(r.vis_lens[0]), int(r.text_lens[0])
+
+    # Inputs: per-layer caches and per-(step, layer) queries, generated on the host.
+    ks, vs_, qs = [], [], []
+    q_host = torch.empty((S, L, B, H, D), dtype=torch.bfloat16)
+    for layer in range(L):
+        li = W.make_layer(r, layer, t_cap=t_cap)
+        q = W.make_queries(r, layer, li, steps=S)
+        ks.append(W.round_to(li.k, r.dtype).to(dev))
+        vs_.append(W.round_to(li.v, r.dtype).to(dev))
+        q_host[:, layer] = W.round_to(q, r.dtype)
+    q_dev = q_host.to(dev)
+    vis_start = torch.tensor(r.vis_starts, dtype=torch.int32, device=dev)
+    vis_len = torch.tensor(r.vis_lens, dtype=torch.int32, device=dev)
+    tl_steps = (torch.tensor(r.text_lens, dtype=torch.int32)[None, :] + torch.arange(S, dtype=torch.int32)[:, None]).to(dev)
+    span = vp.span(vis_start, vis_len)
+    kc = [vp.kv_contiguous(k) for k in ks]
+    vc = [vp.kv_contiguous(v) for v in vs_]
+    budget = vp.make_budget(**r.budget)
+    cfg = vp.make_config(B, H, Hkv, D, nv0, nv0 + tl0 + S, vp.VP_BF16)
+    ctx = vp.vp_init(cfg)
+    cap = vp.vp_max_kept(budget, nv0)
+    out = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
+    kept = torch.empty((L, B, cap), dtype=torch.int32, device=dev)
+    count = torch.zeros((S, L, B), dtype=torch.int32, device=dev)
+    mass = torch.empty((L, B, H), dtype=torch.float32, device=dev)
+    stats = torch.empty((S, L, B, 4), dtype=torch.float32, device=dev)
+
+    def step_calls(s, stream=None):
+        for layer in range(L):
+            vp.vp_decode_step(ctx, B, q_dev[s, layer], kc[layer], vc[layer], span, tl_steps[s], budget,
+                              out[layer], kept[layer], cap, count[s, layer], mass[layer], stats[s, layer],
+                              stream=stream)
+
+    # One eager step loads the kernels; then one CUDA graph per step, with the
+    # stage-timing events of every call captured as graph nodes.
+    step_calls(0)
+    vp.vp_check_errors(ctx)
+    vp.vp_timing_enable(ctx, S * L)
+    graphs = []
+    cap_stream = torch.cuda.Stream(device=dev)
+    for s in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cap_stream):
+            step_calls(s)
+        graphs.append(g)
+    torch.cuda.synchronize()
+
+    for s in range(args.warmup):
+        graphs[s].replay()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    sampler = ClockSampler(dev)
+    sampler.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record()
+    for s in range(args.warmup, S):
+        graphs[s].replay()
+    ev1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+        torch.distributed.barrier()
+    vp.vp_check_errors(ctx)
+
+    # Per-stage device times of the timed calls (events recorded on the calls' stream).
+    stage = vp.vp_timing_read(ctx, S * L)[args.warmup * L:]
+    counts = count.cpu().numpy()
+    score_bytes = gather_bytes = 0
+    for s in range(args.warmup, S):
+        for layer in range(L):
+            for b in range(B):
+                a, c = call_bytes(r, nv0, tl0 + s, int(counts[s, layer, b]))
+                score_bytes += a
+                gather_bytes += c
+    n_calls = args.steps * L
+    score_ms = sum(x[0] for x in stage)
+    select_ms = sum(x[1] for x in stage)
+    gather_ms = sum(x[2] for x in stage)
+    peak, peak_src = measured_peaks()
+    achieved = score_bytes / (score_ms * 1e-3) / 1e9
+    traffic = committed_traffic()
+    ms_per_step = elapsed_ms / args.steps
+    value = world * args.steps / (elapsed_ms * 1e-3)
+    step_gbs = (score_bytes + gather_bytes) / (elapsed_ms * 1e-3) / 1e9
+    kept_frac = float(counts[args.warmup:].mean()) / nv0
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(workload_config(r), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
+        "hbm": {"achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
+                "frac_of_nominal_8tbs": step_gbs / NOMINAL_HBM_GBS,
+                "bytes_per_step": (score_bytes + gather_bytes) / args.steps,
+                "note": "whole step: algorithmic bytes (all visual K + kept visual V + text K/V + q + out) / step time"},
+        "roofline": {"kernel": "k_score", "bound": "hbm", "achieved": achieved, "peak": peak,
+                     "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": traffic,
+                     "avg_launch_us": score_ms * 1e3 / n_calls,
+                     "algorithmic_bytes_per_launch": score_bytes / n_calls},
+        "stages_us_per_call": {"score": score_ms * 1e3 / n_calls, "select": select_ms * 1e3 / n_calls,
+                               "gather": gather_ms * 1e3 / n_calls},
+        "avg_retention": kept_frac,
+        "gpu_launches": 3 * n_calls,
+        "clocks": clocks,
+    }
+    if not args.no_e2e:
+        line["e2e"] = e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, world)
+    if not args.no_cpu_baseline and rank == 0:
+        times = oracle_times("QWEN7B", list(range(4)), args.warmup, args.cpu_seconds, 4 * L)
+        per_call = sum(times) / len(times)
+        line["cpu_baseline"] = {"value": 1.0 / (per_call * L), "unit": UNIT, "cores": 1, "kind": "oracle",
+                                "sample": f"{len(times)} layer calls (layers 0-3, steps from {args.warmup}) "
+                                          f"timed, scaled to a {L}-layer step; single-threaded numpy"}
+    vp.vp_free(ctx)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, world):
+    """Same steps through the C ABI with host buffers: every step copies its
+    queries and the appended token's K/V in from pinned memory, runs the 28
+    layer calls and copies the outputs, kept sets, budgets and masses back."""
+    import torch
+    L, B, H, D = r.layers, r.batch, r.heads, r.head_dim
+    S = args.warmup + args.steps
+    nv0, tl0 = int(r.vis_lens[0]), int(r.text_lens[0])
+    qh = q_host.pin_memory()
+    newk = torch.stack([k[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for k in ks]).cpu().pin_memory()
+    newv = torch.stack([v[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for v in vs_]).cpu().pin_memory()
+    q_in = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
+    tl = torch.empty((B,), dtype=torch.int32, device=dev)
+    tl_host = torch.empty((B,), dtype=torch.int32).pin_memory()
+    out = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
+    kept = torch.empty((L, B, cap), dtype=torch.int32, device=dev)
+    count = torch.empty((L, B), dtype=torch.int32, device=dev)
+    mass = torch.empty((L, B, H), dtype=torch.float32, device=dev)
+    stats = torch.empty((L, B, 4), dtype=torch.float32, device=dev)
+    res = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (out, kept, count, mass, stats)]
+    stream = torch.cuda.current_stream()
+
+    def one(s):
+        pos = nv0 + tl0 - 1 + s
+        tl_host.fill_(tl0 + s)
+        tl.copy_(tl_host, non_blocking=True)
+        q_in.copy_(qh[s], non_blocking=True)
+        for layer in range(L):
+            ks[layer][:, :, pos].copy_(newk[layer][:, :, s], non_blocking=True)
+            vs_[layer][:, :, pos].copy_(newv[layer][:, :, s], non_blocking=True)
+            vp.vp_decode_step(ctx, B, q_in[layer], kc[layer], vc[layer], span, tl, budget, out[layer],
+                              kept[layer], cap, count[layer], mass[layer], stats[layer], stream=stream)
+        for dst, src in zip(res, (out, kept, count, mass, stats)):
+            dst.copy_(src, non_blocking=True)
+        stream.synchronize()
+
+    vp.vp_timing_enable(ctx, 0)
+    for s in range(args.warmup):
+        one(s)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for s in range(args.warmup, S):
+        one(s)
+    el = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([el], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        el = float(t.item())
+    esz = 2
+    h2d = 4 * B + L * B * H * D * esz + 2 * L * B * r.kv_heads * D * esz
+    d2h = sum(t.numel() * t.element_size() for t in (out, kept, count, mass, stats))
+    return {"value": world * args.steps / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": el * 1e3 / args.steps,
+            "note": "direct C-ABI calls (no graph), host wall clock, one stream sync per step"}
+
+
+def committed_traffic():
+    """DRAM bytes per score-kernel launch from the committed ncu summary, if it
+    was taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "score_kernel_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        src = open(os.path.join(ROOT, "paper_2605_31457_gb300", "csrc", "vp_kernels.cu"), "rb").read()
+        if d.get("source_sha256") != hashlib.sha256(src).hexdigest():
+            return None
+        return d.get("dram_bytes_per_launch_full_size")
+    except (OSError, ValueError):
+        return None
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    if world > 1:
+        import torch
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
+    try:
+        return run_ours(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -160,6 +160,22 @@ const char* vp_last_error(const vp_ctx* ctx);
  * vp_last_error) or VP_ERR_CUDA. */
 vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream);
 
+/* Stage timing, for profiling.  vp_timing_enable(ctx, slots) creates
+ * 4 * slots CUDA events owned by the context; from then on the n-th call of
+ * vp_decode_step on the context records, on its own stream, the events of
+ * slot n % slots: before the score kernel and after the score, select and
+ * gather kernels.  Inside stream capture the records become event nodes of
+ * the graph and fire at every replay.  slots = 0 disables timing and releases
+ * the events.  Returns VP_ERR_INVALID_ARG for slots < 0, VP_ERR_CUDA when
+ * event creation fails. */
+vp_status vp_timing_enable(vp_ctx* ctx, int32_t slots);
+
+/* Synchronises the device, then writes for slot s < *n_slots the device time
+ * in milliseconds of stage k (0 score, 1 select, 2 gather) to ms[3 * s + k];
+ * *n_slots = min(max_slots, slots, calls recorded so far).  A slot whose
+ * events have not fired yet reads as a negative value. */
+vp_status vp_timing_read(vp_ctx* ctx, float* ms, int32_t max_slots, int32_t* n_slots);
+
 /* Releases the workspace and the context; NULL is a no-op.  Waits for the
  * device to finish work that may still use the workspace. */
 void vp_free(vp_ctx* ctx);

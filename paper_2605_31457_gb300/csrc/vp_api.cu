@@ -8,6 +8,7 @@
 
 #include <algorithm>
 #include <string>
+#include <vector>
 
 #include "vp.h"
 #include "vp_internal.h"
@@ -27,6 +28,9 @@ struct vp_ctx {
   unsigned* tickets = nullptr;
   unsigned* err = nullptr;
   std::string last_error;
+  std::vector<cudaEvent_t> tev;  // stage-timing events, 4 per slot
+  int32_t tslots = 0;
+  int64_t tcalls = 0;
 };
 
 namespace {
@@ -266,12 +270,26 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
                                                        std::max<int64_t>(1, ceil_div(kept_cap, 16))}));
 
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  cudaError_t e = vp::launch_score(p, st);
+  cudaEvent_t* tev = nullptr;
+  unsigned rec_flags = cudaEventRecordDefault;
+  if (ctx->tslots > 0) {
+    tev = &ctx->tev[4 * (size_t)(ctx->tcalls++ % ctx->tslots)];
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+      rec_flags = cudaEventRecordExternal;
+  }
+  cudaError_t e = cudaSuccess;
+  if (tev) e = cudaEventRecordWithFlags(tev[0], st, rec_flags);
+  if (e == cudaSuccess) e = vp::launch_score(p, st);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: score kernel launch", e);
-  e = vp::launch_select(p, st);
+  if (tev) e = cudaEventRecordWithFlags(tev[1], st, rec_flags);
+  if (e == cudaSuccess) e = vp::launch_select(p, st);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: select kernel launch", e);
-  e = vp::launch_gather(p, st);
+  if (tev) e = cudaEventRecordWithFlags(tev[2], st, rec_flags);
+  if (e == cudaSuccess) e = vp::launch_gather(p, st);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: gather kernel launch", e);
+  if (tev) e = cudaEventRecordWithFlags(tev[3], st, rec_flags);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: timing event", e);
   return VP_OK;
 }
 
@@ -298,8 +316,52 @@ vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream) {
   return fail(ctx, VP_ERR_DEVICE_PRECOND, msg);
 }
 
+vp_status vp_timing_enable(vp_ctx* ctx, int32_t slots) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  if (slots < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_timing_enable: slots < 0");
+  cudaDeviceSynchronize();
+  for (cudaEvent_t ev : ctx->tev) cudaEventDestroy(ev);
+  ctx->tev.clear();
+  ctx->tslots = 0;
+  ctx->tcalls = 0;
+  for (int64_t i = 0; i < 4LL * slots; ++i) {
+    cudaEvent_t ev;
+    cudaError_t e = cudaEventCreate(&ev);
+    if (e != cudaSuccess) {
+      for (cudaEvent_t x : ctx->tev) cudaEventDestroy(x);
+      ctx->tev.clear();
+      return cuda_fail(ctx, "vp_timing_enable: cudaEventCreate", e);
+    }
+    ctx->tev.push_back(ev);
+  }
+  ctx->tslots = slots;
+  return VP_OK;
+}
+
+vp_status vp_timing_read(vp_ctx* ctx, float* ms, int32_t max_slots, int32_t* n_slots) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  if (!ms || !n_slots || max_slots < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_timing_read: bad arguments");
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_timing_read", e);
+  const int64_t n = std::min<int64_t>({(int64_t)max_slots, (int64_t)ctx->tslots, ctx->tcalls});
+  for (int64_t s = 0; s < n; ++s) {
+    for (int k = 0; k < 3; ++k) {
+      float t = -1.f;
+      if (cudaEventElapsedTime(&t, ctx->tev[4 * s + k], ctx->tev[4 * s + k + 1]) != cudaSuccess) t = -1.f;
+      ms[3 * s + k] = t;
+    }
+  }
+  cudaGetLastError();  // an event that never fired leaves a sticky-free error code
+  *n_slots = (int32_t)n;
+  return VP_OK;
+}
+
 void vp_free(vp_ctx* ctx) {
   if (!ctx) return;
+  if (!ctx->tev.empty()) {
+    cudaDeviceSynchronize();
+    for (cudaEvent_t ev : ctx->tev) cudaEventDestroy(ev);
+  }
   if (ctx->ws) cudaFree(ctx->ws);
   delete ctx;
 }

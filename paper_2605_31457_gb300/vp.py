@@ -34,7 +34,8 @@ VP_FIXED_RATIO = 1
 VP_FIXED_K = 2
 VP_DENSE = 3
 
-EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors", "vp_free")
+EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
+            "vp_timing_enable", "vp_timing_read", "vp_free")
 
 
 class vp_config(ctypes.Structure):
@@ -74,6 +75,10 @@ lib.vp_last_error.argtypes = [_P]
 lib.vp_last_error.restype = ctypes.c_char_p
 lib.vp_check_errors.argtypes = [_P, _P]
 lib.vp_check_errors.restype = ctypes.c_int
+lib.vp_timing_enable.argtypes = [_P, ctypes.c_int32]
+lib.vp_timing_enable.restype = ctypes.c_int
+lib.vp_timing_read.argtypes = [_P, ctypes.POINTER(ctypes.c_float), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]
+lib.vp_timing_read.restype = ctypes.c_int
 lib.vp_free.argtypes = [_P]
 lib.vp_free.restype = None
 
@@ -137,6 +142,18 @@ def vp_check_errors(ctx, stream=None, check=True):
         stream = stream.cuda_stream
     st = lib.vp_check_errors(ctx, ctypes.c_void_p(stream))
     return _check(st, ctx) if check else st
+
+
+def vp_timing_enable(ctx, slots: int):
+    return _check(lib.vp_timing_enable(ctx, int(slots)), ctx)
+
+
+def vp_timing_read(ctx, max_slots: int):
+    """Returns a list of (score_ms, select_ms, gather_ms) per recorded slot."""
+    buf = (ctypes.c_float * (3 * max(int(max_slots), 1)))()
+    n = ctypes.c_int32(0)
+    _check(lib.vp_timing_read(ctx, buf, int(max_slots), ctypes.byref(n)), ctx)
+    return [(buf[3 * i], buf[3 * i + 1], buf[3 * i + 2]) for i in range(n.value)]
 
 
 def vp_free(ctx):

@@ -217,6 +217,6 @@ def test_serving_paged_full_size_layer(vp):
 
 @pytest.mark.parametrize("nv", [576, 2304])
 def test_sweep_points(vp, nv):
+    inp = Hn.make_inputs(W.sweep_recipe(nv, W.ADAPTIVE_5PCT))
     for budget in W.SWEEP_BUDGETS:
-        r = W.sweep_recipe(nv, budget)
-        Hn.check_all(vp, Hn.make_inputs(r), budget, seqs=(0, 31, 63))
+        Hn.check_all(vp, inp, budget, seqs=(0, 31, 63))
