@@ -176,6 +176,35 @@ vp_status vp_timing_enable(vp_ctx* ctx, int32_t slots);
  * events have not fired yet reads as a negative value. */
 vp_status vp_timing_read(vp_ctx* ctx, float* ms, int32_t max_slots, int32_t* n_slots);
 
+/* Bytes of the fixed device scratch behind vp_decode_step_noalloc. */
+#define VP_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/* The decode step without a context and without allocating anything.  The
+ * paper has no counterpart: this entry point exists for callers that cannot
+ * allocate device memory on their inference path -- a plugin or custom-op
+ * host whose framework owns all device memory through its own pool, or a
+ * latency-critical loop that must not pay for an allocation.  Arguments mean
+ * what they mean for vp_decode_step, with the static shapes passed as `cfg`.
+ * The intermediate scratch lives in one fixed VP_NOALLOC_SCRATCH_BYTES device
+ * array that every GPU loading the library holds until the process exits:
+ *   - a (cfg, batch) whose scratch would not fit returns VP_ERR_CAPACITY and
+ *     enqueues nothing; malformed arguments return VP_ERR_INVALID_ARG;
+ *   - the first call on each device resolves the array's device address and
+ *     must therefore come before any stream capture on that device;
+ *   - every call shares the array (its counters are cleared at the start of
+ *     each call on `cuda_stream`), so calls whose work overlaps on the GPU --
+ *     on different streams, or from several threads -- race and corrupt each
+ *     other's results; serialise them;
+ *   - device-side range checks still clamp bad spans and skip bad page ids,
+ *     but their flags are not reported (there is no context to read them).
+ * No cudaMalloc, cudaFree or other allocating call is made. */
+vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch, const void* q,
+                                 const vp_kv* k_cache, const vp_kv* v_cache,
+                                 const vp_span* visual_span, const int32_t* text_len,
+                                 const vp_budget* budget, void* out,
+                                 int32_t* kept_idx, int32_t kept_cap, int32_t* kept_count,
+                                 float* mass, float* mass_stats, void* cuda_stream);
+
 /* Releases the workspace and the context; NULL is a no-op.  Waits for the
  * device to finish work that may still use the workspace. */
 void vp_free(vp_ctx* ctx);

@@ -69,6 +69,8 @@ cudaError_t launch_score(const StepParams& p, cudaStream_t s);
 cudaError_t launch_select(const StepParams& p, cudaStream_t s);
 cudaError_t launch_gather(const StepParams& p, cudaStream_t s);
 cudaError_t configure_kernels(int max_visual);
+// Raises (never lowers) the select kernel's dynamic shared-memory limit.
+cudaError_t raise_select_smem(int max_visual);
 size_t select_smem_bytes(int max_visual);
 
 }  // namespace vp

@@ -760,4 +760,13 @@ cudaError_t configure_kernels(int max_visual) {
                               (int)select_smem_bytes(max_visual));
 }
 
+cudaError_t raise_select_smem(int max_visual) {
+  cudaFuncAttributes attr;
+  cudaError_t e = cudaFuncGetAttributes(&attr, k_select);
+  if (e != cudaSuccess) return e;
+  const int need = (int)select_smem_bytes(max_visual);
+  if (attr.maxDynamicSharedSizeBytes >= need) return cudaSuccess;
+  return cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
+}
+
 }  // namespace vp

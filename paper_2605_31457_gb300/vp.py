@@ -35,7 +35,8 @@ VP_FIXED_K = 2
 VP_DENSE = 3
 
 EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
-            "vp_timing_enable", "vp_timing_read", "vp_free")
+            "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc")
+VP_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 class vp_config(ctypes.Structure):
@@ -79,6 +80,10 @@ lib.vp_timing_enable.argtypes = [_P, ctypes.c_int32]
 lib.vp_timing_enable.restype = ctypes.c_int
 lib.vp_timing_read.argtypes = [_P, ctypes.POINTER(ctypes.c_float), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]
 lib.vp_timing_read.restype = ctypes.c_int
+lib.vp_decode_step_noalloc.argtypes = [ctypes.POINTER(vp_config), ctypes.c_int32, _P, ctypes.POINTER(vp_kv),
+                                       ctypes.POINTER(vp_kv), ctypes.POINTER(vp_span), _P,
+                                       ctypes.POINTER(vp_budget), _P, _P, ctypes.c_int32, _P, _P, _P, _P]
+lib.vp_decode_step_noalloc.restype = ctypes.c_int
 lib.vp_free.argtypes = [_P]
 lib.vp_free.restype = None
 
@@ -158,6 +163,23 @@ def vp_timing_read(ctx, max_slots: int):
 
 def vp_free(ctx):
     lib.vp_free(ctx)
+
+
+def vp_decode_step_noalloc(cfg: vp_config, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span: vp_span,
+                           text_len, budget: vp_budget, out, kept_idx, kept_cap, kept_count, mass,
+                           mass_stats=None, stream=None):
+    """The decode step without a context or any device allocation (scratch in
+    the library's fixed device array).  For callers that cannot allocate on
+    their inference path.  Returns the raw vp_status (0 = VP_OK)."""
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream().cuda_stream
+    elif hasattr(stream, "cuda_stream"):
+        stream = stream.cuda_stream
+    return lib.vp_decode_step_noalloc(ctypes.byref(cfg), int(batch), _ptr(q), ctypes.byref(k_cache),
+                                      ctypes.byref(v_cache), ctypes.byref(visual_span), _ptr(text_len),
+                                      ctypes.byref(budget), _ptr(out), _ptr(kept_idx), int(kept_cap),
+                                      _ptr(kept_count), _ptr(mass), _ptr(mass_stats), ctypes.c_void_p(stream))
 
 
 # ------------------------------------------------------- marshalling helpers
