@@ -17,7 +17,7 @@ struct vp_ctx {
   vp_config cfg;
   int device = 0;
   int num_sms = 0;
-  int ns_max = 1, nk_max = 1;
+  vp::WsLayout lay;
   void* ws = nullptr;
   size_t ws_bytes = 0;
   float* z_ws = nullptr;
@@ -25,6 +25,8 @@ struct vp_ctx {
   float* split_o = nullptr;
   float* gpart_o = nullptr;
   float* gpart_st = nullptr;
+  float* mt_o = nullptr;
+  float* mt_st = nullptr;
   unsigned* tickets = nullptr;
   unsigned* err = nullptr;
   std::string last_error;
@@ -56,7 +58,6 @@ int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Largest K_t the budget yields for n visual tokens (K_t is non-decreasing in
 // N_v in every mode, so the bound for max_visual covers every sequence).
@@ -158,28 +159,10 @@ vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx) {
     delete ctx;
     return st;
   }
-  const int H = c.num_q_heads, Hkv = c.num_kv_heads, G = H / Hkv, D = c.head_dim;
-  // Split counts: enough CTAs for a batch of one sequence to cover every SM
-  // four times, and at least 32 work units (tokens) per split.
-  const int64_t work_max = (int64_t)c.max_visual + 2LL * c.max_seq;
-  ctx->ns_max = (int)std::max<int64_t>(1, std::min<int64_t>({256, ceil_div(4LL * ctx->num_sms, Hkv), ceil_div(work_max, 32)}));
-  ctx->nk_max = (int)std::max<int64_t>(1, std::min<int64_t>(64, ceil_div(2LL * ctx->num_sms, Hkv)));
-
-  const size_t B = (size_t)c.max_batch;
-  const size_t sz_z = B * H * (size_t)std::max(c.max_visual, 1) * 4;
-  const size_t sz_st = B * H * (size_t)ctx->ns_max * vp::ST_N * 4;
-  const size_t sz_o = B * H * (size_t)ctx->ns_max * D * 4;
-  const size_t sz_go = B * Hkv * (size_t)ctx->nk_max * G * D * 4;
-  const size_t sz_gs = B * Hkv * (size_t)ctx->nk_max * G * 2 * 4;
-  const size_t sz_t = B * Hkv * 4;
-  size_t off = 0;
-  const size_t o_z = off; off = round_up(off + sz_z, 256);
-  const size_t o_st = off; off = round_up(off + sz_st, 256);
-  const size_t o_o = off; off = round_up(off + sz_o, 256);
-  const size_t o_go = off; off = round_up(off + sz_go, 256);
-  const size_t o_gs = off; off = round_up(off + sz_gs, 256);
-  const size_t o_t = off; off = round_up(off + sz_t, 256);
-  const size_t o_e = off; off = round_up(off + 4, 256);
+  ctx->lay = vp::ws_layout(c.max_batch, c.num_q_heads, c.num_kv_heads, c.head_dim, c.max_visual, c.max_seq,
+                          ctx->num_sms);
+  const vp::WsLayout& L = ctx->lay;
+  const size_t off = L.total;
   ctx->ws_bytes = off;
   e = cudaMalloc(&ctx->ws, ctx->ws_bytes);
   if (e != cudaSuccess) {
@@ -188,15 +171,17 @@ vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx) {
     return st;
   }
   char* base = static_cast<char*>(ctx->ws);
-  ctx->z_ws = reinterpret_cast<float*>(base + o_z);
-  ctx->split_st = reinterpret_cast<float*>(base + o_st);
-  ctx->split_o = reinterpret_cast<float*>(base + o_o);
-  ctx->gpart_o = reinterpret_cast<float*>(base + o_go);
-  ctx->gpart_st = reinterpret_cast<float*>(base + o_gs);
-  ctx->tickets = reinterpret_cast<unsigned*>(base + o_t);
-  ctx->err = reinterpret_cast<unsigned*>(base + o_e);
+  ctx->z_ws = reinterpret_cast<float*>(base + L.o_z);
+  ctx->split_st = reinterpret_cast<float*>(base + L.o_st);
+  ctx->split_o = reinterpret_cast<float*>(base + L.o_o);
+  ctx->gpart_o = reinterpret_cast<float*>(base + L.o_go);
+  ctx->gpart_st = reinterpret_cast<float*>(base + L.o_gs);
+  ctx->mt_o = reinterpret_cast<float*>(base + L.o_mo);
+  ctx->mt_st = reinterpret_cast<float*>(base + L.o_ms);
+  ctx->tickets = reinterpret_cast<unsigned*>(base + L.o_tickets);
+  ctx->err = reinterpret_cast<unsigned*>(base + L.o_err);
   e = cudaMemset(ctx->ws, 0, ctx->ws_bytes);
-  if (e == cudaSuccess) e = vp::configure_kernels(c.max_visual);
+  if (e == cudaSuccess) e = vp::configure_kernels(c.max_visual, c.num_q_heads, L.nsp_max);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) {
     vp_status st = cuda_fail(nullptr, "vp_init: workspace set-up failed", e);
@@ -263,11 +248,12 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   p.mass = mass; p.mass_stats = mass_stats;
   p.z_ws = ctx->z_ws; p.split_st = ctx->split_st; p.split_o = ctx->split_o;
   p.gpart_o = ctx->gpart_o; p.gpart_st = ctx->gpart_st; p.tickets = ctx->tickets; p.err = ctx->err;
-  p.ns_max = ctx->ns_max; p.nk_max = ctx->nk_max;
-  const int64_t units = (int64_t)batch * Hkv;
-  p.ns = (int)std::max<int64_t>(1, std::min<int64_t>(ctx->ns_max, ceil_div(4LL * ctx->num_sms, units)));
-  p.nk = (int)std::max<int64_t>(1, std::min<int64_t>({(int64_t)ctx->nk_max, ceil_div(2LL * ctx->num_sms, units),
-                                                       std::max<int64_t>(1, ceil_div(kept_cap, 16))}));
+  const vp::Plan pl = vp::make_plan(batch, Hkv, c.head_dim, ctx->num_sms, c.max_visual, c.max_seq, kept_cap,
+                                    budget->granularity);
+  p.hp = ctx->lay.hp;
+  p.ns = pl.ns; p.nsp_max = ctx->lay.nsp_max; p.cl = pl.cl;
+  p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
+  p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st;
 
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   cudaEvent_t* tev = nullptr;
@@ -313,6 +299,7 @@ vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream) {
   if (word & vp::ERR_PAGE) msg += " block table entry outside the pool;";
   if (word & vp::ERR_KEPT) msg += " kept index outside the visual span;";
   if (word & vp::ERR_NONFINITE) msg += " non-finite importance score;";
+  if (word & vp::ERR_TIMEOUT) msg += " an asynchronous copy did not complete in time;";
   return fail(ctx, VP_ERR_DEVICE_PRECOND, msg);
 }
 

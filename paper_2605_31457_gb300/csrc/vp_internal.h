@@ -14,12 +14,14 @@ enum : unsigned {
   ERR_LEN = 4u,        // vis_len + text_len > max_seq
   ERR_PAGE = 8u,       // block-table entry outside [0, num_pages) or row past max_pages
   ERR_KEPT = 16u,      // a kept index outside [0, N_v)
-  ERR_NONFINITE = 32u  // a non-finite score reached the selection
+  ERR_NONFINITE = 32u, // a non-finite score reached the selection
+  ERR_TIMEOUT = 64u    // a bounded wait for an asynchronous copy gave up
 };
 
 // Split statistics written by the score kernel for every (sequence, query
-// head, split); maxima are in log2 units (z * log2 e).
-enum { ST_MV = 0, ST_L1V, ST_LTV, ST_MT, ST_L1T, ST_LTT, ST_N };
+// head, split), padded to two float4; maxima are in log2 units (z * log2 e).
+// The text half comes first: the gather kernel reads only that float4.
+enum { ST_MT = 0, ST_L1T = 1, ST_LTT = 2, ST_MV = 4, ST_L1V = 5, ST_LTV = 6, ST_N = 8 };
 
 struct KvView {
   const void* data;
@@ -53,24 +55,96 @@ struct StepParams {
   float* mass;
   float* mass_stats;
   // workspace
-  float* z_ws;        // [max_batch][H][max_visual] visual logits, log2 units
-  float* split_st;    // [max_batch][H][ns_max][ST_N]
-  float* split_o;     // [max_batch][H][ns_max][D]  text partial outputs
+  float* z_ws;        // [max_batch][max_visual][hp] visual logits, log2 units
+  float* split_st;    // [max_batch][H][nsp_max][ST_N] (one partial per cluster of splits)
+  float* split_o;     // [max_batch][H][nsp_max][D]    text partial outputs
   float* gpart_o;     // [max_batch][Hkv][nk_max][G][D] kept-visual partial outputs
   float* gpart_st;    // [max_batch][Hkv][nk_max][G][2] {max, sum}
+  float* mt_o;        // [max_batch][H][D] text output merged over the splits
+  float* mt_st;       // [max_batch][H][2] its {max, sum}
   unsigned* tickets;  // [max_batch][Hkv] (zero between calls)
   unsigned* err;      // device error word
-  int ns, ns_max;     // score splits used by this call / allocated
+  int hp;             // z_ws row stride (H rounded up to a multiple of 4)
+  int ns, nsp_max;    // score splits (= text partials) per (sequence, kv-head); allocated
+  int cl;             // CTAs in a select cluster
   int nk, nk_max;     // gather chunks used by this call / allocated
+  int nm;             // gather CTAs that also merge a slice of the text partials (0: ns == 1)
+  int nc;             // gather CTAs per (sequence, kv-head) = max(nk, nm)
+  int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= 256)
 };
+
+// ---------------------------------------------------------------- host planning
+
+constexpr int kNkMax = 64;    // kept chunks per (sequence, kv-head)
+constexpr int kNsMax = 256;   // score splits per (sequence, kv-head)
+constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
+
+// Launch plan of one call: about one score CTA per SM when the batch is small,
+// select clusters that spread the importance scores of few sequences over
+// several SMs, gather chunks of about 256 kept rows.
+struct Plan {
+  int ns, cl, nk, nm, nc, gslice;
+};
+
+inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, int max_seq, int kept_cap,
+                      int granularity) {
+  const long long units = (long long)batch * Hkv;
+  const long long tiles = (max_visual + 15) / 16 + 2LL * ((max_seq + 15) / 16);  // work of the longest sequence
+  long long ns = (num_sms + units - 1) / units;
+  const long long ns_work = tiles / 8 > 1 ? tiles / 8 : 1;  // keep a few tiles per warp
+  if (ns > ns_work) ns = ns_work;
+  if (ns > kNsMax) ns = kNsMax;
+  if (ns < 1) ns = 1;
+  const long long sel = (long long)batch * (granularity ? Hkv : 1);
+  int cl = 1;
+  while (cl < 8 && sel * cl * 2 <= num_sms) cl *= 2;
+  long long nk = (kept_cap + 255) / 256;
+  if (nk < 1) nk = 1;
+  if (nk > kNkMax) nk = kNkMax;
+  const int nm = ns > 1 ? (D / 16 < kMaxMerge ? D / 16 : kMaxMerge) : 0;
+  return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), kept_cap <= 256 ? 1 : 0};
+}
+
+// Workspace layout for up to `batch` sequences (offsets in bytes, 256-aligned).
+// The first `zero_bytes` (tickets, error word) must be zero before a call.
+struct WsLayout {
+  size_t o_tickets, o_err, zero_bytes, o_z, o_st, o_o, o_go, o_gs, o_mo, o_ms, total;
+  int hp, nsp_max, nk_max;
+};
+
+inline size_t ws_round(size_t x) { return (x + 255) / 256 * 256; }
+
+inline WsLayout ws_layout(int batch, int H, int Hkv, int D, int max_visual, int max_seq, int num_sms) {
+  WsLayout w;
+  w.hp = (H + 3) / 4 * 4;
+  w.nk_max = kNkMax;
+  w.nsp_max = 1;
+  for (int bb = 1; bb <= batch; ++bb) {
+    const Plan pl = make_plan(bb, Hkv, D, num_sms, max_visual, max_seq, 0, 0);
+    if (pl.ns > w.nsp_max) w.nsp_max = pl.ns;
+  }
+  const size_t B = (size_t)batch, G = (size_t)(H / Hkv);
+  size_t off = 0;
+  w.o_tickets = off; off = ws_round(off + B * Hkv * 4);
+  w.o_err = off; off = ws_round(off + 4);
+  w.zero_bytes = off;
+  w.o_z = off; off = ws_round(off + B * (size_t)(max_visual > 0 ? max_visual : 1) * w.hp * 4);
+  w.o_st = off; off = ws_round(off + B * H * (size_t)w.nsp_max * ST_N * 4);
+  w.o_o = off; off = ws_round(off + B * H * (size_t)w.nsp_max * D * 4);
+  w.o_go = off; off = ws_round(off + B * Hkv * (size_t)w.nk_max * G * D * 4);
+  w.o_gs = off; off = ws_round(off + B * Hkv * (size_t)w.nk_max * G * 2 * 4);
+  w.o_mo = off; off = ws_round(off + B * H * (size_t)D * 4);
+  w.o_ms = off; off = ws_round(off + B * H * 2 * 4);
+  w.total = off;
+  return w;
+}
 
 // Launchers (vp_kernels.cu).  Return the launch error, if any.
 cudaError_t launch_score(const StepParams& p, cudaStream_t s);
 cudaError_t launch_select(const StepParams& p, cudaStream_t s);
 cudaError_t launch_gather(const StepParams& p, cudaStream_t s);
-cudaError_t configure_kernels(int max_visual);
-// Raises (never lowers) the select kernel's dynamic shared-memory limit.
-cudaError_t raise_select_smem(int max_visual);
-size_t select_smem_bytes(int max_visual);
+// Kernel attributes: raises (never lowers) the select kernel's dynamic
+// shared-memory limit for these shapes and sets the other kernels' limits.
+cudaError_t configure_kernels(int max_visual, int H, int nsp_max);
 
 }  // namespace vp

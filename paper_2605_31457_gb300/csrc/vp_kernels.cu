@@ -2,40 +2,58 @@
 //
 //   k_score   per (sequence, kv-head, split): logits of the G query heads of the
 //             kv-head against every key of the split (Eq. 6's Z).  Visual logits
-//             go to the workspace; visual and text tokens get separate online
+//             go to the workspace; visual and text tokens keep separate online
 //             softmax statistics at tau = 1 and at tau (the two sums of Eq. 6);
 //             text tokens also accumulate their unnormalised attention output.
-//   k_select  per sequence (or per kv-head): merges the split statistics into
-//             the visual mass per head (Eq. 5) and its head-max (Sec. 4.3), the
-//             budget K_t (Eq. 7 + clamp of Sec. 5.2), the importance score S_i
-//             (Eq. 2) and the Top-K_t set (Eq. 3) by radix select, ties to the
+//   k_select  per sequence (or per kv-head), a cluster of up to 8 CTAs: merges
+//             the split statistics into the visual mass per head (Eq. 5) and
+//             its head-max (Sec. 4.3) and the budget K_t (Eq. 7 + clamp of
+//             Sec. 5.2); every CTA computes the importance score S_i (Eq. 2) of
+//             a slice of the visual tokens into rank 0's shared memory, which
+//             then finds the Top-K_t set (Eq. 3) by radix select, ties to the
 //             lower index, emitted in ascending order.
-//   k_gather  per (sequence, kv-head, chunk of the kept set): attention of the
-//             kept visual tokens, reading V only for them; the last chunk to
-//             finish merges every partial (text splits and kept chunks) in
+//   k_gather  per (sequence, kv-head): CTA c attends over chunk c of the kept
+//             visual tokens, reading V only for them, and merges slice c of the
+//             text partials; the last CTA to finish combines everything in
 //             log-sum-exp form and writes the output (Sec. 4.2, Sec. 5.7).
 //
 // Logits are carried in log2 units (z * log2 e) so that every exponential is
-// one exp2f; exp(z - m) = exp2(z2 - m2) and exp((z - m) / tau) =
-// exp2((z2 - m2) / tau).
-#include <cuda_runtime.h>
+// one exp2f: exp(z - m) = exp2(z2 - m2), exp((z - m) / tau) = exp2((z2 - m2) / tau).
+//
+// Every kernel starts with griddepcontrol.wait, so it may be launched as a
+// programmatic dependent of the preceding kernel on the stream: it reads no
+// input before that kernel has completed and its writes are visible.
+#include <cooperative_groups.h>
 #include <cuda_bf16.h>
+#include <cuda_runtime.h>
 #include <math_constants.h>
 #include <stdint.h>
 
 #include "vp_internal.h"
 
+namespace cg = cooperative_groups;
+
 namespace vp {
 namespace {
 
-constexpr int kWarps = 4;
+constexpr int kWarps = 4;                 // warps of a score CTA
 constexpr int kThreads = 32 * kWarps;
+constexpr int kStages = 3;                // TMA ring depth per warp
+constexpr int kTile = 16;                 // tokens per tile
 constexpr int kSelThreads = 1024;
 constexpr int kMaxHeads = 128;
-constexpr int kGatherTile = 64;  // kept tokens staged per round in k_gather
+constexpr int kGatherThreads = 256;
+constexpr int kGatherWarps = kGatherThreads / 32;
+constexpr int kGatherTile = 64;           // kept tokens staged per round in k_gather
+constexpr long long kSpinLimit = 1LL << 22;  // mbarrier polls before a wait gives up
 
 // Budget modes (numbering of vp_budget_mode in include/vp.h).
 enum { MODE_ADAPTIVE = 0, MODE_FIXED_RATIO = 1, MODE_FIXED_K = 2, MODE_DENSE = 3 };
+
+// ------------------------------------------------------------------ helpers
+
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 __device__ __forceinline__ float warp_max(float x) {
 #pragma unroll
@@ -47,6 +65,17 @@ __device__ __forceinline__ float warp_sum(float x) {
   for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
   return x;
 }
+// Reductions over the 8 lanes that share lane % 4 (the mma "group" axis).
+__device__ __forceinline__ float group_max(float x) {
+  x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 4));
+  x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 8));
+  return fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 16));
+}
+__device__ __forceinline__ float group_sum(float x) {
+  x += __shfl_xor_sync(0xffffffffu, x, 4);
+  x += __shfl_xor_sync(0xffffffffu, x, 8);
+  return x + __shfl_xor_sync(0xffffffffu, x, 16);
+}
 
 // exp2(a - m) with an empty term (a = -inf) giving exactly 0.
 __device__ __forceinline__ float exp2_rel(float a, float m) {
@@ -56,8 +85,6 @@ __device__ __forceinline__ float exp2_tau(float a, float m, float inv_tau) {
   return a == -CUDART_INF_F ? 0.f : exp2f((a - m) * inv_tau);
 }
 
-__device__ __forceinline__ float to_f(float x) { return x; }
-__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
 template <typename T> __device__ __forceinline__ T from_f(float x);
 template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
 template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float x) {
@@ -69,10 +96,10 @@ template <int N>
 __device__ __forceinline__ void load_f(const float* p, float (&f)[N]) {
   static_assert(N == 1 || N == 2 || N == 4, "fp32 vector width");
   if constexpr (N == 4) {
-    float4 v = __ldg(reinterpret_cast<const float4*>(p));
+    const float4 v = __ldg(reinterpret_cast<const float4*>(p));
     f[0] = v.x; f[1] = v.y; f[2] = v.z; f[3] = v.w;
   } else if constexpr (N == 2) {
-    float2 v = __ldg(reinterpret_cast<const float2*>(p));
+    const float2 v = __ldg(reinterpret_cast<const float2*>(p));
     f[0] = v.x; f[1] = v.y;
   } else {
     f[0] = __ldg(p);
@@ -86,15 +113,77 @@ template <int N>
 __device__ __forceinline__ void load_f(const __nv_bfloat16* p, float (&f)[N]) {
   static_assert(N == 2 || N == 4 || N == 8, "bf16 vector width");
   if constexpr (N == 8) {
-    uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+    const uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
     bf2(v.x, f[0], f[1]); bf2(v.y, f[2], f[3]); bf2(v.z, f[4], f[5]); bf2(v.w, f[6], f[7]);
   } else if constexpr (N == 4) {
-    uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
+    const uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
     bf2(v.x, f[0], f[1]); bf2(v.y, f[2], f[3]);
   } else {
-    uint32_t v = __ldg(reinterpret_cast<const unsigned int*>(p));
-    bf2(v, f[0], f[1]);
+    bf2(__ldg(reinterpret_cast<const unsigned int*>(p)), f[0], f[1]);
   }
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+  return r;
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+// D = A * B + D, m16n8k16, bf16 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ unsigned smem_u32(const void* p) {
+  return static_cast<unsigned>(__cvta_generic_to_shared(p));
+}
+// Four 8x8 b16 matrices from shared memory; lane l gives the row address of
+// row l % 8 of matrix l / 8.
+__device__ __forceinline__ void ldsm_x4(unsigned addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(unsigned addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+
+// ---- mbarrier + bulk (TMA) copies
+__device__ __forceinline__ void mbar_init(uint64_t* bar, unsigned count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() { asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory"); }
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, unsigned bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
+  unsigned ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Bounded wait for a phase of an mbarrier; false if it never completed.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
+  for (long long i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (i > 32) __nanosleep(64);
+  }
+  return false;
+}
+// Orders this thread's earlier generic-proxy shared-memory accesses before
+// later asynchronous-proxy (bulk copy) writes to the same memory.
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, unsigned bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
 
 struct Seq {
@@ -128,62 +217,418 @@ __device__ __forceinline__ const T* kv_row(const KvView& kv, const StepParams& p
   return base + (int64_t)page * kv.sb + (int64_t)g * kv.sh + (int64_t)(pos & (p.page_size - 1)) * kv.st;
 }
 
-// Raw dot products of one key row with the GM (padded) query heads in shared memory.
-template <typename T, int D, int GM>
-__device__ __forceinline__ void dot_row(const T* row, const float (*q_s)[D], float (&z)[GM]) {
-  constexpr int CH = 16 / sizeof(T);
+// Token ranges of split s: the sequence's work (visual tokens weigh 1, text
+// tokens 2) cut into ns equal parts.  Visual range [va, vb) is relative to the
+// span start; text range [ta, tb) indexes the text tokens in cache order.
+struct SplitRange {
+  int va, vb, ta, tb;
+};
+__device__ __forceinline__ SplitRange split_range(const Seq& sq, int s, int ns) {
+  const int W = sq.nv + 2 * sq.tl;
+  const int per = (W + ns - 1) / ns;
+  const int w0 = min(W, s * per), w1 = min(W, w0 + per);
+  SplitRange r;
+  r.va = min(w0, sq.nv);
+  r.vb = min(w1, sq.nv);
+  r.ta = (max(w0, sq.nv) - sq.nv + 1) >> 1;
+  r.tb = (max(w1, sq.nv) - sq.nv + 1) >> 1;
+  return r;
+}
+__device__ __forceinline__ int text_pos(const Seq& sq, int ti) { return ti < sq.vs ? ti : ti + sq.nv; }
+
+// Merges n statistic records (`stride` floats apart); writes the text weight of
+// each record to wt[k * wstride].
+__device__ __forceinline__ void merge_stats(const float* recs, int n, int stride, float inv_tau, float* out,
+                                            float* wt, int wstride) {
+  float Mv = -CUDART_INF_F, Mt = -CUDART_INF_F;
+  for (int k = 0; k < n; ++k) {
+    Mv = fmaxf(Mv, recs[k * stride + ST_MV]);
+    Mt = fmaxf(Mt, recs[k * stride + ST_MT]);
+  }
+  float l1v = 0.f, ltv = 0.f, l1t = 0.f, ltt = 0.f;
+  for (int k = 0; k < n; ++k) {
+    const float* r = recs + k * stride;
+    l1v += exp2_rel(r[ST_MV], Mv) * r[ST_L1V];
+    ltv += exp2_tau(r[ST_MV], Mv, inv_tau) * r[ST_LTV];
+    const float at = exp2_rel(r[ST_MT], Mt);
+    l1t += at * r[ST_L1T];
+    ltt += exp2_tau(r[ST_MT], Mt, inv_tau) * r[ST_LTT];
+    wt[k * wstride] = at;
+  }
+  out[ST_MT] = Mt; out[ST_L1T] = l1t; out[ST_LTT] = ltt; out[3] = 0.f;
+  out[ST_MV] = Mv; out[ST_L1V] = l1v; out[ST_LTV] = ltv; out[7] = 0.f;
+}
+
+// ------------------------------------------------------- score epilogue
+// Shared by both score kernels: per-warp statistics wst[w][h][ST_N] and text
+// outputs (warp w at ow + w * ow_stride, [GM][D]) are merged into the CTA's
+// partial and written to split slot s.
+template <int GM, int D>
+struct ScoreTail {
+  float cst[GM][ST_N];
+  float wsc[kWarps][GM];
+};
+
+template <int GM, int D>
+__device__ void score_epilogue(const StepParams& p, int b, int g, int s, const float (*wst)[GM][ST_N],
+                               const float* ow, int ow_stride, ScoreTail<GM, D>& tl) {
+  const int tid = threadIdx.x, G = p.G;
+  constexpr int D4 = D / 4;
+  __syncthreads();
+  if (tid < G) merge_stats(&wst[0][tid][0], kWarps, GM * ST_N, p.inv_tau, tl.cst[tid], &tl.wsc[0][tid], GM);
+  __syncthreads();
+  const int64_t rec0 = ((int64_t)b * p.H + g * G) * p.nsp_max + s;  // slot of head 0
+  for (int i = tid; i < G * D4; i += kThreads) {
+    const int h = i / D4, d = 4 * (i % D4);
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-  for (int h = 0; h < GM; ++h) z[h] = 0.f;
-#pragma unroll 4
-  for (int d0 = 0; d0 < D; d0 += CH) {
-    float kf[CH];
-    load_f<CH>(row + d0, kf);
-#pragma unroll
-    for (int h = 0; h < GM; ++h) {
-#pragma unroll
-      for (int e = 0; e < CH; e += 4) {
-        const float4 qv = *reinterpret_cast<const float4*>(&q_s[h][d0 + e]);
-        z[h] = fmaf(qv.x, kf[e], z[h]);
-        z[h] = fmaf(qv.y, kf[e + 1], z[h]);
-        z[h] = fmaf(qv.z, kf[e + 2], z[h]);
-        z[h] = fmaf(qv.w, kf[e + 3], z[h]);
-      }
+    for (int w = 0; w < kWarps; ++w) {
+      const float a = tl.wsc[w][h];
+      const float4 v = *reinterpret_cast<const float4*>(ow + w * ow_stride + h * D + d);
+      o.x = fmaf(a, v.x, o.x); o.y = fmaf(a, v.y, o.y); o.z = fmaf(a, v.z, o.z); o.w = fmaf(a, v.w, o.w);
     }
+    *reinterpret_cast<float4*>(p.split_o + (rec0 + (int64_t)h * p.nsp_max) * D + d) = o;
+  }
+  if (tid < 2 * G) {
+    const int h = tid >> 1, half = tid & 1;
+    *reinterpret_cast<float4*>(p.split_st + (rec0 + (int64_t)h * p.nsp_max) * ST_N + 4 * half) =
+        *reinterpret_cast<const float4*>(&tl.cst[h][4 * half]);
   }
 }
 
 // ---------------------------------------------------------------------------
-// k_score: grid (ns, Hkv, B), 128 threads.  Each warp walks 32-token groups
-// (lane = token) of the split; a split covers a slice of the sequence's work,
-// visual tokens weighing 1 (K only) and text tokens 2 (K and V).
+// k_score_mma (bf16).  Each warp streams 16-token tiles through a 3-stage ring
+// in shared memory: one lane arms the stage's mbarrier with the tile's byte
+// count, then lane r issues a bulk (TMA) copy of token row r of K (and of V
+// for text tiles) into a row padded to 2D + 16 bytes, which makes the
+// ldmatrix reads below free of bank conflicts.  Both contractions run on the
+// tensor cores with mma.m16n8k16:
+//   QK:  A = K tile (16 tokens x 16 dims, ldmatrix), B = q^T (16 dims x 8 heads).
+//   PV:  A = V^T (16 dims x 16 tokens, ldmatrix.trans), B = P^T (16 tokens x
+//        8 heads), taken from the QK accumulators with four shuffles.
+// Lane (r = lane/4, c = lane%4) keeps the softmax statistics of heads 2c, 2c+1
+// of each 8-head tile and accumulates the same heads' outputs, so rescaling
+// the accumulators needs no communication.
 // ---------------------------------------------------------------------------
-template <typename T, int D, int GM>
-__global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
-  constexpr int DPL = D / 32;  // dims per lane in the text P.V phase
+template <int D, int NT>
+struct MmaCfg {
+  static constexpr int GM = 8 * NT;
+  static constexpr int KS = D / 16;                    // QK k-steps
+  static constexpr int MT = D / 16;                    // PV m-tiles (16 dims each)
+  static constexpr int RP = 2 * D + 16;                // padded row pitch (bytes)
+  static constexpr int TILE_BYTES = kTile * RP;
+  static constexpr int STAGE = 2 * TILE_BYTES;         // K tile + V tile
+  static constexpr int RING = kStages * STAGE;         // per warp
+  static constexpr int OFF_BAR = kWarps * RING;
+  static constexpr int OFF_TAIL = OFF_BAR + kWarps * kStages * 8;
+  static constexpr int OFF_WST = OFF_TAIL + (int)sizeof(ScoreTail<GM, D>);
+  static constexpr size_t SMEM = (size_t)OFF_WST + sizeof(float) * kWarps * GM * ST_N;
+  static_assert(GM * D * 4 <= RING, "a warp's text partial must fit in its ring");
+  static_assert(OFF_TAIL % 16 == 0 && OFF_WST % 16 == 0, "alignment");
+};
+
+template <int D, int NT>
+__global__ void __launch_bounds__(kThreads) k_score_mma(const __grid_constant__ StepParams p) {
+  using C = MmaCfg<D, NT>;
+  constexpr int GM = C::GM;
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gr = lane >> 2, tg = lane & 3;  // mma group id / thread in group
+  const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  unsigned char* ring = smem + warp * C::RING;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + warp * kStages;
+  auto& tail = *reinterpret_cast<ScoreTail<GM, D>*>(smem + C::OFF_TAIL);
+  auto wst = reinterpret_cast<float (*)[GM][ST_N]>(smem + C::OFF_WST);
+
+  if (lane == 0) {
+    for (int i = 0; i < kStages; ++i) mbar_init(bars + i, 1);
+    mbar_fence_init();
+  }
+  __syncwarp();
+  pdl_wait();
+  const int G = p.G, H = p.H;
+  const Seq sq = load_seq(p, b, s == 0 && g == 0);
+  const SplitRange rg = split_range(sq, s, p.ns);
+  const int n_vt = (rg.vb - rg.va + kTile - 1) / kTile;
+  const int n_tt = (rg.tb - rg.ta + kTile - 1) / kTile;
+  const int n_tiles = n_vt + n_tt;
+  const int my_n = warp < n_tiles ? (n_tiles - warp + kWarps - 1) / kWarps : 0;
+
+  unsigned err = 0;
+  int issued = 0;  // tiles whose copies were issued
+  // Arms stage k % kStages and issues the bulk copies of this warp's k-th tile.
+  auto issue = [&](int k) {
+    if (k >= my_n) return;
+    issued = k + 1;
+    const int j = warp + kWarps * k;
+    const bool text = j >= n_vt;
+    const int first = text ? rg.ta + (j - n_vt) * kTile : rg.va + j * kTile;
+    const int cnt = min(kTile, (text ? rg.tb : rg.vb) - first);
+    uint64_t* bar = bars + k % kStages;
+    unsigned char* kt = ring + (k % kStages) * C::STAGE;
+    const __nv_bfloat16* kr = nullptr;
+    const __nv_bfloat16* vr = nullptr;
+    if (lane < cnt) {
+      const int pos = text ? text_pos(sq, first + lane) : sq.vs + first + lane;
+      kr = kv_row<__nv_bfloat16>(p.k, p, b, g, pos);
+      if (text) vr = kv_row<__nv_bfloat16>(p.v, p, b, g, pos);
+      if (!kr || (text && !vr)) { err |= ERR_PAGE; kr = vr = nullptr; }
+    }
+    const unsigned nk = __popc(__ballot_sync(0xffffffffu, kr != nullptr));
+    const unsigned nvr = __popc(__ballot_sync(0xffffffffu, vr != nullptr));
+    fence_proxy_async();
+    if (lane == 0) mbar_expect_tx(bar, (nk + nvr) * (2 * D));
+    __syncwarp();
+    if (kr) bulk_g2s(kt + lane * C::RP, kr, 2 * D, bar);
+    if (vr) bulk_g2s(kt + C::TILE_BYTES + lane * C::RP, vr, 2 * D, bar);
+  };
+#pragma unroll
+  for (int k = 0; k < kStages - 1; ++k) issue(k);
+
+  // q^T fragments (natural dimension order): head 8n + gr, dims 16ks + 2tg (+8).
+  uint32_t qf[NT][C::KS][2];
+  const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(p.q) + ((int64_t)b * H + g * G) * D;
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+    const int h = 8 * n + gr;
+    const uint32_t* qr = reinterpret_cast<const uint32_t*>(qb + h * D);
+#pragma unroll
+    for (int ks = 0; ks < C::KS; ++ks) {
+      qf[n][ks][0] = h < G ? __ldg(qr + 8 * ks + tg) : 0u;
+      qf[n][ks][1] = h < G ? __ldg(qr + 8 * ks + 4 + tg) : 0u;
+    }
+  }
+
+  float m_v[NT][2], l1v[NT][2], ltv[NT][2], m_t[NT][2], l1t[NT][2], ltt[NT][2];
+  float acc[NT][C::MT][4];
+#pragma unroll
+  for (int n = 0; n < NT; ++n) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      m_v[n][j] = m_t[n][j] = -CUDART_INF_F;
+      l1v[n][j] = ltv[n][j] = l1t[n][j] = ltt[n][j] = 0.f;
+    }
+#pragma unroll
+    for (int mi = 0; mi < C::MT; ++mi)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[n][mi][e] = 0.f;
+  }
+
+  // ldmatrix row addresses.  K (A operand, rows = tokens): matrix l / 8 covers
+  // tokens 8 * ((l / 8) & 1) + (0..7) and dims 8 * (l / 16) + (0..7) of the 16 x 16
+  // block.  V^T (A operand via .trans, rows = dims): matrix l / 8 covers
+  // tokens 8 * (l / 16) + (0..7) and dims 8 * ((l / 8) & 1) + (0..7).
+  const int krow = (lane & 7) + 8 * ((lane >> 3) & 1), kcol = 8 * (lane >> 4);
+  const int vrow = (lane & 7) + 8 * (lane >> 4), vcol = 8 * ((lane >> 3) & 1);
+  bool timed_out = false;
+  int consumed = 0;  // tiles whose copies were waited for
+  for (int k = 0; k < my_n; ++k) {
+    if (!mbar_wait(bars + k % kStages, (k / kStages) & 1)) { timed_out = true; break; }
+    consumed = k + 1;
+    const int j = warp + kWarps * k;
+    const bool text = j >= n_vt;
+    const int first = text ? rg.ta + (j - n_vt) * kTile : rg.va + j * kTile;
+    const int cnt = min(kTile, (text ? rg.tb : rg.vb) - first);
+    const unsigned kt = smem_u32(ring + (k % kStages) * C::STAGE);
+    const unsigned vt = kt + C::TILE_BYTES;
+
+    // ---- QK on the tensor cores
+    float c[NT][4];
+#pragma unroll
+    for (int n = 0; n < NT; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) c[n][e] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < C::KS; ++ks) {
+      uint32_t a0, a1, a2, a3;
+      ldsm_x4(kt + krow * C::RP + (16 * ks + kcol) * 2, a0, a1, a2, a3);
+#pragma unroll
+      for (int n = 0; n < NT; ++n) mma_bf16(c[n], a0, a1, a2, a3, qf[n][ks][0], qf[n][ks][1]);
+    }
+    // c[n][e]: token row gr + 8 * (e >> 1), head 8n + 2tg + (e & 1).  Rows past
+    // cnt were not copied (stale shared memory): they are masked here.
+    const bool ok0 = gr < cnt, ok1 = gr + 8 < cnt;
+    float zz[NT][4];
+#pragma unroll
+    for (int n = 0; n < NT; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const bool ok = (e < 2 ? ok0 : ok1) && (8 * n + 2 * tg + (e & 1)) < G;
+        zz[n][e] = ok ? c[n][e] * p.c_log2 : -CUDART_INF_F;
+      }
+
+    if (!text) {
+      float* zrow = p.z_ws + ((int64_t)b * p.max_visual + first) * p.hp + g * G;
+#pragma unroll
+      for (int n = 0; n < NT; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int h = 8 * n + 2 * tg + (e & 1), r = gr + 8 * (e >> 1);
+          if (h < G && r < cnt) zrow[(int64_t)r * p.hp + h] = zz[n][e];
+        }
+#pragma unroll
+      for (int n = 0; n < NT; ++n)
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          const float mn = fmaxf(m_v[n][jj], group_max(fmaxf(zz[n][jj], zz[n][jj + 2])));
+          if (mn > m_v[n][jj]) {
+            l1v[n][jj] *= exp2_rel(m_v[n][jj], mn);
+            ltv[n][jj] *= exp2_tau(m_v[n][jj], mn, p.inv_tau);
+            m_v[n][jj] = mn;
+          }
+          if (mn != -CUDART_INF_F) {
+            l1v[n][jj] += exp2f(zz[n][jj] - mn) + exp2f(zz[n][jj + 2] - mn);
+            ltv[n][jj] += exp2f((zz[n][jj] - mn) * p.inv_tau) + exp2f((zz[n][jj + 2] - mn) * p.inv_tau);
+          }
+        }
+    } else {
+      uint32_t pb[NT][2];
+#pragma unroll
+      for (int n = 0; n < NT; ++n) {
+        float pr[4];
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          const float mn = fmaxf(m_t[n][jj], group_max(fmaxf(zz[n][jj], zz[n][jj + 2])));
+          if (mn > m_t[n][jj]) {
+            const float a = exp2_rel(m_t[n][jj], mn);
+            l1t[n][jj] *= a;
+            ltt[n][jj] *= exp2_tau(m_t[n][jj], mn, p.inv_tau);
+#pragma unroll
+            for (int mi = 0; mi < C::MT; ++mi) {
+              acc[n][mi][jj] *= a;
+              acc[n][mi][jj + 2] *= a;
+            }
+            m_t[n][jj] = mn;
+          }
+          pr[jj] = pr[jj + 2] = 0.f;
+          if (mn != -CUDART_INF_F) {
+            pr[jj] = exp2f(zz[n][jj] - mn);
+            pr[jj + 2] = exp2f(zz[n][jj + 2] - mn);
+            l1t[n][jj] += pr[jj] + pr[jj + 2];
+            ltt[n][jj] += exp2f((zz[n][jj] - mn) * p.inv_tau) + exp2f((zz[n][jj + 2] - mn) * p.inv_tau);
+          }
+        }
+        // P^T fragment for head 8n + gr: tokens 2tg, 2tg + 1 live in the first
+        // halves of lanes 8tg + gr/2 and 8tg + 4 + gr/2, tokens 2tg + 8, 2tg + 9
+        // in their second halves; the half is chosen by the head's parity.
+        const uint32_t p01 = pack_bf16(pr[0], pr[1]), p23 = pack_bf16(pr[2], pr[3]);
+        const int src0 = 8 * tg + (gr >> 1), src1 = src0 + 4;
+        const uint32_t x0 = __shfl_sync(0xffffffffu, p01, src0), x1 = __shfl_sync(0xffffffffu, p01, src1);
+        const uint32_t x2 = __shfl_sync(0xffffffffu, p23, src0), x3 = __shfl_sync(0xffffffffu, p23, src1);
+        const uint32_t sel = (gr & 1) ? 0x7632u : 0x5410u;
+        pb[n][0] = prmt(x0, x1, sel);
+        pb[n][1] = prmt(x2, x3, sel);
+      }
+      // ---- PV on the tensor cores.  V rows past cnt hold stale data: their
+      // probabilities are 0, but a stale NaN would still poison the product, so
+      // the fragment words of those rows are zeroed.
+      const bool vok_lo0 = 2 * tg < cnt, vok_lo1 = 2 * tg + 1 < cnt;
+      const bool vok_hi0 = 2 * tg + 8 < cnt, vok_hi1 = 2 * tg + 9 < cnt;
+      const bool full = cnt == kTile;
+#pragma unroll
+      for (int mi = 0; mi < C::MT; ++mi) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4_t(vt + vrow * C::RP + (16 * mi + vcol) * 2, a0, a1, a2, a3);
+        if (!full) {
+          // a0/a1: tokens 2tg (low half), 2tg + 1 (high half); a2/a3: tokens 2tg + 8, 2tg + 9.
+          const uint32_t mlo = (vok_lo0 ? 0x0000ffffu : 0u) | (vok_lo1 ? 0xffff0000u : 0u);
+          const uint32_t mhi = (vok_hi0 ? 0x0000ffffu : 0u) | (vok_hi1 ? 0xffff0000u : 0u);
+          a0 &= mlo; a1 &= mlo; a2 &= mhi; a3 &= mhi;
+        }
+#pragma unroll
+        for (int n = 0; n < NT; ++n) mma_bf16(acc[n][mi], a0, a1, a2, a3, pb[n][0], pb[n][1]);
+      }
+    }
+    __syncwarp();
+    issue(k + kStages - 1);
+  }
+  // After a timed-out wait, the copies still in flight must land (or time out
+  // again) before the ring is reused for the partials or the CTA exits.
+  for (int k = consumed; k < issued; ++k)
+    if (!mbar_wait(bars + k % kStages, (k / kStages) & 1)) timed_out = true;
+  pdl_trigger();
+  if (timed_out) err |= ERR_TIMEOUT;
+  if (err) atomicOr(p.err, err);
+
+  // Warp partials: statistics to wst, text outputs into this warp's (now idle) ring.
+#pragma unroll
+  for (int n = 0; n < NT; ++n)
+#pragma unroll
+    for (int jj = 0; jj < 2; ++jj) {
+      const float a = group_sum(l1v[n][jj]), bb = group_sum(ltv[n][jj]);
+      const float cc = group_sum(l1t[n][jj]), dd = group_sum(ltt[n][jj]);
+      const int h = 8 * n + 2 * tg + jj;
+      if (gr == 0) {
+        wst[warp][h][ST_MV] = m_v[n][jj]; wst[warp][h][ST_L1V] = a; wst[warp][h][ST_LTV] = bb;
+        wst[warp][h][ST_MT] = m_t[n][jj]; wst[warp][h][ST_L1T] = cc; wst[warp][h][ST_LTT] = dd;
+        wst[warp][h][3] = wst[warp][h][7] = 0.f;
+      }
+    }
+  // acc[n][mi]: rows (dims) 16mi + gr and 16mi + gr + 8, heads 8n + 2tg, 8n + 2tg + 1.
+  float* ow = reinterpret_cast<float*>(ring);
+#pragma unroll
+  for (int n = 0; n < NT; ++n)
+#pragma unroll
+    for (int mi = 0; mi < C::MT; ++mi) {
+      const int h0 = 8 * n + 2 * tg, d0 = 16 * mi + gr;
+      ow[h0 * D + d0] = acc[n][mi][0];
+      ow[(h0 + 1) * D + d0] = acc[n][mi][1];
+      ow[h0 * D + d0 + 8] = acc[n][mi][2];
+      ow[(h0 + 1) * D + d0 + 8] = acc[n][mi][3];
+    }
+  score_epilogue<GM, D>(p, b, g, s, wst, reinterpret_cast<const float*>(smem), C::RING / 4, tail);
+}
+
+// ---------------------------------------------------------------------------
+// k_score_f32 (fp32 caches): lane-per-token dot products on the FMA pipes,
+// lane-per-dimension P.V; the same partials as k_score_mma.
+// ---------------------------------------------------------------------------
+template <int D, int GM>
+struct F32Smem {
+  float q[GM][D];
+  float pr[kWarps][GM][32];
+  const float* vrow[kWarps][32];
+  float wst[kWarps][GM][ST_N];
+  float ow[kWarps][GM][D];
+  ScoreTail<GM, D> tail;
+};
+
+template <int D, int GM>
+__device__ __forceinline__ void dot_row_f32(const float* row, const float (*q_s)[D], float (&z)[GM]) {
+#pragma unroll
+  for (int h = 0; h < GM; ++h) z[h] = 0.f;
+#pragma unroll 4
+  for (int d0 = 0; d0 < D; d0 += 4) {
+    float kf[4];
+    load_f<4>(row + d0, kf);
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      const float4 qv = *reinterpret_cast<const float4*>(&q_s[h][d0]);
+      z[h] = fmaf(qv.x, kf[0], z[h]);
+      z[h] = fmaf(qv.y, kf[1], z[h]);
+      z[h] = fmaf(qv.z, kf[2], z[h]);
+      z[h] = fmaf(qv.w, kf[3], z[h]);
+    }
+  }
+}
+
+template <int D, int GM>
+__global__ void __launch_bounds__(kThreads) k_score_f32(const __grid_constant__ StepParams p) {
+  constexpr int DPL = D / 32;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  auto& sm = *reinterpret_cast<F32Smem<D, GM>*>(smem_raw);
   const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_wait();
   const int G = p.G, H = p.H;
-
-  __shared__ __align__(16) float q_s[GM][D];
-  __shared__ float pr_s[kWarps][GM][32];
-  __shared__ const T* vrow_s[kWarps][32];
-  __shared__ float wst_s[kWarps][GM][ST_N];
-  __shared__ float wsc_s[kWarps][GM];
-  __shared__ __align__(16) float o_s[GM][D];
-
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
-  const T* qb = reinterpret_cast<const T*>(p.q) + ((int64_t)b * H + g * G) * D;
+  const float* qb = reinterpret_cast<const float*>(p.q) + ((int64_t)b * H + g * G) * D;
   for (int i = threadIdx.x; i < GM * D; i += kThreads) {
     const int h = i / D, d = i % D;
-    q_s[h][d] = h < G ? to_f(qb[h * D + d]) : 0.f;
+    sm.q[h][d] = h < G ? qb[h * D + d] : 0.f;
   }
   __syncthreads();
-
-  const int W = sq.nv + 2 * sq.tl;
-  const int per = (W + p.ns - 1) / p.ns;
-  const int w0 = min(W, s * per), w1 = min(W, w0 + per);
-  const int va = min(w0, sq.nv), vb = min(w1, sq.nv);
-  const int ta = (max(w0, sq.nv) - sq.nv + 1) >> 1, tb = (max(w1, sq.nv) - sq.nv + 1) >> 1;
+  const SplitRange rg = split_range(sq, s, p.ns);
 
   float m_v[GM], l1v[GM], ltv[GM], m_t[GM], l1t[GM], ltt[GM], acc[GM][DPL];
 #pragma unroll
@@ -195,20 +640,19 @@ __global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
   }
   unsigned err = 0;
 
-  // Visual tokens: logits to the workspace, visual statistics.
-  for (int base = va + warp * 32; base < vb; base += kWarps * 32) {
+  for (int base = rg.va + warp * 32; base < rg.vb; base += kWarps * 32) {
     const int i = base + lane;
-    bool valid = i < vb;
+    bool valid = i < rg.vb;
     float z[GM];
     if (valid) {
-      const T* row = kv_row<T>(p.k, p, b, g, sq.vs + i);
-      if (row) dot_row<T, D, GM>(row, q_s, z); else { valid = false; err |= ERR_PAGE; }
+      const float* row = kv_row<float>(p.k, p, b, g, sq.vs + i);
+      if (row) dot_row_f32<D, GM>(row, sm.q, z); else { valid = false; err |= ERR_PAGE; }
     }
 #pragma unroll
     for (int h = 0; h < GM; ++h) {
       if (h >= G) break;
       const float zz = valid ? z[h] * p.c_log2 : -CUDART_INF_F;
-      if (i < vb) p.z_ws[((int64_t)b * H + g * G + h) * p.max_visual + i] = zz;
+      if (i < rg.vb) p.z_ws[((int64_t)b * p.max_visual + i) * p.hp + g * G + h] = zz;
       const float mn = fmaxf(m_v[h], warp_max(zz));
       if (mn > m_v[h]) {
         l1v[h] *= exp2_rel(m_v[h], mn);
@@ -222,17 +666,16 @@ __global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
     }
   }
 
-  // Text tokens: text statistics and the unnormalised text output.
-  for (int base = ta + warp * 32; base < tb; base += kWarps * 32) {
+  for (int base = rg.ta + warp * 32; base < rg.tb; base += kWarps * 32) {
     const int ti = base + lane;
-    bool valid = ti < tb;
-    const int pos = ti < sq.vs ? ti : ti + sq.nv;
+    bool valid = ti < rg.tb;
+    const int pos = text_pos(sq, ti);
     float z[GM];
-    const T* vrow = nullptr;
+    const float* vrow = nullptr;
     if (valid) {
-      const T* row = kv_row<T>(p.k, p, b, g, pos);
-      vrow = kv_row<T>(p.v, p, b, g, pos);
-      if (row && vrow) dot_row<T, D, GM>(row, q_s, z); else { valid = false; vrow = nullptr; err |= ERR_PAGE; }
+      const float* row = kv_row<float>(p.k, p, b, g, pos);
+      vrow = kv_row<float>(p.v, p, b, g, pos);
+      if (row && vrow) dot_row_f32<D, GM>(row, sm.q, z); else { valid = false; vrow = nullptr; err |= ERR_PAGE; }
     }
 #pragma unroll
     for (int h = 0; h < GM; ++h) {
@@ -253,16 +696,16 @@ __global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
         l1t[h] += pr;
         ltt[h] += exp2f((zz - mn) * p.inv_tau);
       }
-      pr_s[warp][h][lane] = pr;
+      sm.pr[warp][h][lane] = pr;
     }
-    vrow_s[warp][lane] = vrow;
+    sm.vrow[warp][lane] = vrow;
     __syncwarp();
-    const int nt = min(32, tb - base);
+    const int nt = min(32, rg.tb - base);
     for (int t0 = 0; t0 < nt; t0 += 4) {
       float vv[4][DPL];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const T* vr = t0 + u < nt ? vrow_s[warp][t0 + u] : nullptr;
+        const float* vr = t0 + u < nt ? sm.vrow[warp][t0 + u] : nullptr;
         if (vr) load_f<DPL>(vr + lane * DPL, vv[u]);
         else {
 #pragma unroll
@@ -274,7 +717,7 @@ __global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
 #pragma unroll
         for (int h = 0; h < GM; ++h) {
           if (h >= G) break;
-          const float pr = t0 + u < nt ? pr_s[warp][h][t0 + u] : 0.f;
+          const float pr = t0 + u < nt ? sm.pr[warp][h][t0 + u] : 0.f;
 #pragma unroll
           for (int j = 0; j < DPL; ++j) acc[h][j] = fmaf(pr, vv[u][j], acc[h][j]);
         }
@@ -282,65 +725,28 @@ __global__ void __launch_bounds__(kThreads) k_score(const StepParams p) {
     }
     __syncwarp();
   }
+  pdl_trigger();
   if (err) atomicOr(p.err, err);
 
-  // Merge the four warps: statistics, then the text outputs (fixed order).
 #pragma unroll
   for (int h = 0; h < GM; ++h) {
-    if (h >= G) break;
     const float a = warp_sum(l1v[h]), bb = warp_sum(ltv[h]);
     const float c = warp_sum(l1t[h]), d = warp_sum(ltt[h]);
     if (lane == 0) {
-      wst_s[warp][h][ST_MV] = m_v[h]; wst_s[warp][h][ST_L1V] = a; wst_s[warp][h][ST_LTV] = bb;
-      wst_s[warp][h][ST_MT] = m_t[h]; wst_s[warp][h][ST_L1T] = c; wst_s[warp][h][ST_LTT] = d;
+      sm.wst[warp][h][ST_MV] = m_v[h]; sm.wst[warp][h][ST_L1V] = a; sm.wst[warp][h][ST_LTV] = bb;
+      sm.wst[warp][h][ST_MT] = m_t[h]; sm.wst[warp][h][ST_L1T] = c; sm.wst[warp][h][ST_LTT] = d;
+      sm.wst[warp][h][3] = sm.wst[warp][h][7] = 0.f;
     }
-  }
-  __syncthreads();
-  if (threadIdx.x < G) {
-    const int h = threadIdx.x;
-    float Mv = -CUDART_INF_F, Mt = -CUDART_INF_F;
-    for (int w = 0; w < kWarps; ++w) {
-      Mv = fmaxf(Mv, wst_s[w][h][ST_MV]);
-      Mt = fmaxf(Mt, wst_s[w][h][ST_MT]);
-    }
-    float r[ST_N] = {Mv, 0.f, 0.f, Mt, 0.f, 0.f};
-    for (int w = 0; w < kWarps; ++w) {
-      const float mv = wst_s[w][h][ST_MV], mt = wst_s[w][h][ST_MT];
-      r[ST_L1V] += exp2_rel(mv, Mv) * wst_s[w][h][ST_L1V];
-      r[ST_LTV] += exp2_tau(mv, Mv, p.inv_tau) * wst_s[w][h][ST_LTV];
-      const float at = exp2_rel(mt, Mt);
-      r[ST_L1T] += at * wst_s[w][h][ST_L1T];
-      r[ST_LTT] += exp2_tau(mt, Mt, p.inv_tau) * wst_s[w][h][ST_LTT];
-      wsc_s[w][h] = at;
-    }
-    float* dst = p.split_st + (((int64_t)b * H + g * G + h) * p.ns_max + s) * ST_N;
 #pragma unroll
-    for (int k = 0; k < ST_N; ++k) dst[k] = r[k];
+    for (int j = 0; j < DPL; ++j) sm.ow[warp][h][lane * DPL + j] = acc[h][j];
   }
-  __syncthreads();
-  for (int w = 0; w < kWarps; ++w) {
-    if (warp == w) {
-#pragma unroll
-      for (int h = 0; h < GM; ++h) {
-        if (h >= G) break;
-#pragma unroll
-        for (int j = 0; j < DPL; ++j) {
-          const float prev = w == 0 ? 0.f : o_s[h][lane * DPL + j];
-          o_s[h][lane * DPL + j] = fmaf(wsc_s[w][h], acc[h][j], prev);
-        }
-      }
-    }
-    __syncthreads();
-  }
-  for (int i = threadIdx.x; i < G * D; i += kThreads) {
-    const int h = i / D, d = i % D;
-    p.split_o[(((int64_t)b * H + g * G + h) * p.ns_max + s) * D + d] = o_s[h][d];
-  }
+  score_epilogue<GM, D>(p, b, g, s, sm.wst, &sm.ow[0][0][0], GM * D, sm.tail);
 }
 
 // ---------------------------------------------------------------------------
-// k_select: grid (granularity ? Hkv : 1, B), 1024 threads, dynamic shared
-// memory holding the N_v score keys.
+// k_select: grid (cl, granularity ? Hkv : 1, B) in clusters of cl CTAs,
+// 1024 threads.  Dynamic shared memory: rank 0 holds the N_v score keys; every
+// rank stages the split statistics after them.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int budget_k(const StepParams& p, float m_max, int nv) {
   if (nv <= 0) return 0;
@@ -389,40 +795,112 @@ __device__ __forceinline__ int block_excl_scan(int x, int* wsum_s) {
   return res;
 }
 
-__global__ void __launch_bounds__(kSelThreads) k_select(const StepParams p) {
-  extern __shared__ uint32_t key_s[];
+__global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ StepParams p) {
+  extern __shared__ __align__(16) uint32_t key_s[];  // [max_visual] keys, then [H][ns][ST_N] statistics
   __shared__ float hM_s[kMaxHeads], hInv_s[kMaxHeads], hMass_s[kMaxHeads], hMass1_s[kMaxHeads];
   __shared__ unsigned hist_s[256];
   __shared__ int wsum_s[32];
   __shared__ int sh_i[4];
 
-  const int gsel = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  const int H = p.H;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
+  pdl_wait();
+  pdl_trigger();
+  const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31;
+  const int H = p.H, ns = p.ns;
   const Seq sq = load_seq(p, b, false);
   const int nv = sq.nv;
+  float* st_s = reinterpret_cast<float*>(key_s + ((p.max_visual + 3) & ~3));
 
-  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5, Eq. 6).
-  for (int h = tid; h < H; h += kSelThreads) {
-    const float* st = p.split_st + ((int64_t)b * H + h) * p.ns_max * ST_N;
+  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5, Eq. 6):
+  //    staged with one parallel load, then merged per head.
+  for (int i = tid; i < H * ns * 2; i += kSelThreads) {
+    const int h = i / (2 * ns), sp = (i >> 1) % ns, half = i & 1;
+    *reinterpret_cast<float4*>(st_s + (h * ns + sp) * ST_N + 4 * half) = __ldcg(
+        reinterpret_cast<const float4*>(p.split_st + (((int64_t)b * H + h) * p.nsp_max + sp) * ST_N + 4 * half));
+  }
+  // The first logit row of this thread's slice is fetched now, while the
+  // statistics are still in flight (heads up to 32).
+  const int per = (nv + ncl - 1) / ncl;
+  const int i0 = min(nv, rank * per), i1 = min(nv, i0 + per);
+  const int hbeg = p.granularity ? gsel * p.G : 0;
+  const int hcnt = p.granularity ? p.G : H;
+  const bool vec = (hbeg & 3) == 0 && (hcnt & 3) == 0;
+  const bool pre = vec && hcnt <= 32 && i0 + tid < i1;
+  float4 zpre[8];
+  if (pre) {
+    const float4* zr = reinterpret_cast<const float4*>(p.z_ws + ((int64_t)b * p.max_visual + i0 + tid) * p.hp + hbeg);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) zpre[q] = 4 * q < hcnt ? __ldcg(zr + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
+  // One warp per head, lanes over the splits.
+  for (int h = tid >> 5; h < H; h += kSelThreads / 32) {
+    const float* st = st_s + h * ns * ST_N;
     float M = -CUDART_INF_F;
-    for (int s = 0; s < p.ns; ++s) M = fmaxf(M, fmaxf(st[s * ST_N + ST_MV], st[s * ST_N + ST_MT]));
+    for (int s = lane; s < ns; s += 32) M = fmaxf(M, fmaxf(st[s * ST_N + ST_MV], st[s * ST_N + ST_MT]));
+    M = warp_max(M);
     float L1v = 0.f, L1t = 0.f, Ltv = 0.f, Ltt = 0.f;
-    for (int s = 0; s < p.ns; ++s) {
+    for (int s = lane; s < ns; s += 32) {
       const float* r = st + s * ST_N;
       L1v += exp2_rel(r[ST_MV], M) * r[ST_L1V];
       Ltv += exp2_tau(r[ST_MV], M, p.inv_tau) * r[ST_LTV];
       L1t += exp2_rel(r[ST_MT], M) * r[ST_L1T];
       Ltt += exp2_tau(r[ST_MT], M, p.inv_tau) * r[ST_LTT];
     }
-    const float L1 = L1v + L1t, Lt = Ltv + Ltt;
-    hM_s[h] = M;
-    hInv_s[h] = L1 > 0.f ? 1.f / L1 : 0.f;
-    hMass_s[h] = Lt > 0.f ? Ltv / Lt : 0.f;
-    hMass1_s[h] = L1 > 0.f ? L1v / L1 : 0.f;
+    L1v = warp_sum(L1v); Ltv = warp_sum(Ltv); L1t = warp_sum(L1t); Ltt = warp_sum(Ltt);
+    if (lane == 0) {
+      const float L1 = L1v + L1t, Lt = Ltv + Ltt;
+      hM_s[h] = M;
+      hInv_s[h] = L1 > 0.f ? 1.f / L1 : 0.f;
+      hMass_s[h] = Lt > 0.f ? Ltv / Lt : 0.f;
+      hMass1_s[h] = L1 > 0.f ? L1v / L1 : 0.f;
+    }
   }
   __syncthreads();
 
-  // 2. Head mean, head max (Sec. 4.3) and the budget (Eq. 7).
+  // 2. Importance S_i (Eq. 2) of this rank's slice of the visual tokens, as
+  //    float bits (S >= 0 orders like its bits), into rank 0's key array.
+  const float inv_cnt = 1.f / (float)hcnt;
+  uint32_t* key0 = ncl > 1 ? cluster.map_shared_rank(key_s, 0) : key_s;
+  unsigned bad = 0;
+  for (int i = i0 + tid; i < i1; i += kSelThreads) {
+    const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
+    float a = 0.f;
+    if (pre && i == i0 + tid) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (4 * q < hcnt) {
+          const int h = hbeg + 4 * q;
+          a = fmaf(exp2_rel(zpre[q].x, hM_s[h]), hInv_s[h], a);
+          a = fmaf(exp2_rel(zpre[q].y, hM_s[h + 1]), hInv_s[h + 1], a);
+          a = fmaf(exp2_rel(zpre[q].z, hM_s[h + 2]), hInv_s[h + 2], a);
+          a = fmaf(exp2_rel(zpre[q].w, hM_s[h + 3]), hInv_s[h + 3], a);
+        }
+      }
+    } else if (vec) {
+      for (int hh = 0; hh < hcnt; hh += 4) {
+        const float4 z4 = __ldcg(reinterpret_cast<const float4*>(zr + hh));
+        const int h = hbeg + hh;
+        a = fmaf(exp2_rel(z4.x, hM_s[h]), hInv_s[h], a);
+        a = fmaf(exp2_rel(z4.y, hM_s[h + 1]), hInv_s[h + 1], a);
+        a = fmaf(exp2_rel(z4.z, hM_s[h + 2]), hInv_s[h + 2], a);
+        a = fmaf(exp2_rel(z4.w, hM_s[h + 3]), hInv_s[h + 3], a);
+      }
+    } else {
+      for (int hh = 0; hh < hcnt; ++hh)
+        a = fmaf(exp2_rel(__ldcg(zr + hh), hM_s[hbeg + hh]), hInv_s[hbeg + hh], a);
+    }
+    const float sc = a * inv_cnt;
+    if (!isfinite(sc)) bad = 1;
+    key0[i] = __float_as_uint(sc);
+  }
+  if (bad) atomicOr(p.err, ERR_NONFINITE);
+  if (ncl > 1) cluster.sync();  // rank 0 now sees every key
+  else __syncthreads();
+  if (rank != 0) return;
+
+  // 3. Head mean, head max (Sec. 4.3) and the budget (Eq. 7).
   if (tid < 32) {
     float sm = 0.f, mx = 0.f, s1 = 0.f;
     for (int h = tid; h < H; h += 32) {
@@ -446,44 +924,40 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const StepParams p) {
   }
   if (gsel == 0)
     for (int h = tid; h < H; h += kSelThreads) p.mass[(int64_t)b * H + h] = hMass_s[h];
-
-  // 3. Importance S_i (Eq. 2), kept as float bits (S >= 0 orders like its bits).
-  const int hbeg = p.granularity ? gsel * p.G : 0;
-  const int hcnt = p.granularity ? p.G : H;
   __syncthreads();
   const int K = sh_i[0];
-  unsigned bad = 0;
-  for (int i = tid; i < nv; i += kSelThreads) {
-    float a = 0.f;
-    for (int hh = 0; hh < hcnt; ++hh) {
-      const int h = hbeg + hh;
-      const float z = p.z_ws[((int64_t)b * H + h) * p.max_visual + i];
-      a = fmaf(exp2_rel(z, hM_s[h]), hInv_s[h], a);
-    }
-    const float sc = a / (float)hcnt;
-    if (!isfinite(sc)) bad = 1;
-    key_s[i] = __float_as_uint(sc);
-  }
-  if (bad) atomicOr(p.err, ERR_NONFINITE);
-
   const int nsel = p.granularity ? p.Hkv : 1;
   int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
   if (tid == 0) p.kept_count[(int64_t)b * nsel + gsel] = K;
-  __syncthreads();
 
-  // 4. Radix select of the K-th largest key, 8 bits per pass from the top.
+  // 4. Radix select of the K-th largest key, 8 bits per pass from the top;
+  //    lanes holding the same digit add to the histogram once per warp.
   const bool take_all = K >= nv;
   uint32_t theta = 0;
-  unsigned krem = 0;
+  unsigned krem = 0, n_theta = 0;  // keys equal to theta: to keep, in total
   if (K > 0 && !take_all) {
     uint32_t prefix = 0, mask = 0;
     krem = (unsigned)K;
     for (int shift = 24; shift >= 0; shift -= 8) {
       for (int i = tid; i < 256; i += kSelThreads) hist_s[i] = 0;
       __syncthreads();
-      for (int i = tid; i < nv; i += kSelThreads) {
-        const uint32_t k = key_s[i];
-        if ((k & mask) == prefix) atomicAdd(&hist_s[(k >> shift) & 255u], 1u);
+      for (int base = 0; base < nv; base += kSelThreads) {
+        const int i = base + tid;
+        const uint32_t k = i < nv ? key_s[i] : 0u;
+        const bool m = i < nv && (k & mask) == prefix;
+        const unsigned dg = (k >> shift) & 255u;
+        // One atomic per warp when all its candidates share the digit (the
+        // common case in the upper passes); one per lane otherwise.
+        const unsigned act = __ballot_sync(0xffffffffu, m);
+        if (act) {
+          const int leader = __ffs(act) - 1;
+          const unsigned d0 = __shfl_sync(0xffffffffu, dg, leader);
+          if (__all_sync(0xffffffffu, !m || dg == d0)) {
+            if (lane == leader) atomicAdd(&hist_s[d0], (unsigned)__popc(act));
+          } else if (m) {
+            atomicAdd(&hist_s[dg], 1u);
+          }
+        }
       }
       __syncthreads();
       if (tid < 32) {
@@ -511,23 +985,27 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const StepParams p) {
       krem -= (unsigned)sh_i[2];
       prefix |= (uint32_t)sh_i[1] << shift;
       mask |= 255u << shift;
+      if (shift == 0) n_theta = hist_s[sh_i[1]];
       __syncthreads();
     }
     theta = prefix;  // the K-th largest key; krem keys equal to it are kept
   }
 
-  // 5. Ascending compaction: keys above theta, plus the first krem equal keys.
+  // 5. Ascending compaction: keys above theta, plus the first krem equal keys
+  //    (every equal key when there is no tie to break: one scan less).
   if (K > 0) {
-    const int per = (nv + kSelThreads - 1) / kSelThreads;
-    const int i0 = min(nv, tid * per), i1 = min(nv, i0 + per);
+    const int per_t = (nv + kSelThreads - 1) / kSelThreads;
+    const int j0 = min(nv, tid * per_t), j1 = min(nv, j0 + per_t);
+    const bool ties = !take_all && krem < n_theta;
     int n_eq = 0;
-    if (!take_all)
-      for (int i = i0; i < i1; ++i) n_eq += key_s[i] == theta;
-    const int eq_before = block_excl_scan(n_eq, wsum_s);
+    if (ties)
+      for (int i = j0; i < j1; ++i) n_eq += key_s[i] == theta;
+    const int eq_before = ties ? block_excl_scan(n_eq, wsum_s) : 0;
+    if (!ties) krem = 0xffffffffu;
     int n_sel = 0;
     {
       int r = eq_before;
-      for (int i = i0; i < i1; ++i) {
+      for (int i = j0; i < j1; ++i) {
         const uint32_t k = key_s[i];
         const bool sel = take_all || k > theta || (k == theta && (unsigned)r < krem);
         r += k == theta;
@@ -536,7 +1014,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const StepParams p) {
     }
     int o = block_excl_scan(n_sel, wsum_s);
     int r = eq_before;
-    for (int i = i0; i < i1; ++i) {
+    for (int i = j0; i < j1; ++i) {
       const uint32_t k = key_s[i];
       const bool sel = take_all || k > theta || (k == theta && (unsigned)r < krem);
       r += k == theta;
@@ -547,198 +1025,543 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const StepParams p) {
 }
 
 // ---------------------------------------------------------------------------
-// k_gather: grid (nk, Hkv, B), 128 threads.  Chunk c of the kept list is
-// staged 64 tokens at a time: indices, V-row addresses and logits to shared
-// memory, then every thread accumulates one 16-byte slice of the V rows of
-// every (128 / slices-per-row)-th token.  The last chunk of (b, kv-head) to
-// finish merges all partials and writes the output.
+// k_gather: grid (nc, Hkv, B), 256 threads.  CTA c (a) attends over chunk c of
+// the kept list (c < nk), staged 64 tokens at a time -- indices, V-row
+// addresses and logits to shared memory, then each thread accumulates a
+// 16-byte slice of the V rows of every (256 / slices-per-row)-th token -- and
+// (b) merges dimension slice c of the text partials of the score splits
+// (c < nm).  The last CTA of (sequence, kv-head) to finish combines the merged
+// text output with the kept chunks and writes out.
 // ---------------------------------------------------------------------------
 template <typename T, int D, int GM>
-__global__ void __launch_bounds__(kThreads) k_gather(const StepParams p) {
+struct GatherSmem {
+  const T* vrow[kGatherTile];
+  float pz[GM][kGatherTile];
+  float run[GM][4];                         // running max, sum, rescale factor
+  float red[kGatherWarps / 2][GM][D];       // warp-tree reduction buffer
+  float tw[GM][kNsMax];                     // text-split maxima, then weights
+  float tl[GM][kNsMax];                     // text-split sums
+  float fin[GM][4];
+  int last;
+};
+
+template <typename T, int D, int GM>
+__global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant__ StepParams p) {
   constexpr int CH = 16 / sizeof(T);          // elements per 16-byte slice
   constexpr int CPR = D / CH;                 // slices per row
-  constexpr int SLOTS = kThreads / CPR;       // tokens processed side by side
-  static_assert(kThreads % CPR == 0, "row slicing");
+  constexpr int SLOTS = kGatherThreads / CPR; // tokens processed side by side
+  constexpr int D4 = D / 4;
+  static_assert(kGatherThreads % CPR == 0 && CPR <= 32, "row slicing");
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  auto& sm = *reinterpret_cast<GatherSmem<T, D, GM>*>(smem_raw);
   const int c = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int G = p.G, H = p.H;
   const int slot = tid / CPR, ch = tid % CPR;
 
-  __shared__ const T* vrow_s[kGatherTile];
-  __shared__ float pz_s[GM][kGatherTile];
-  __shared__ float run_s[GM][3];  // running max, running sum, rescale factor
-  __shared__ __align__(16) float o_s[GM][D];
-  __shared__ float fin_s[GM];
-  __shared__ int last_s;
-
-  const Seq sq = load_seq(p, b, false);
-  const int sel = p.granularity ? b * p.Hkv + g : b;
-  const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
-  const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
-  const int per = (K + p.nk - 1) / max(p.nk, 1);
-  const int j0 = min(K, c * per), j1 = min(K, j0 + per);
-
-  if (tid < GM) { run_s[tid][0] = -CUDART_INF_F; run_s[tid][1] = 0.f; run_s[tid][2] = 0.f; }
-  float acc[GM][CH];
-#pragma unroll
-  for (int h = 0; h < GM; ++h)
-#pragma unroll
-    for (int e = 0; e < CH; ++e) acc[h][e] = 0.f;
+  pdl_wait();
+  pdl_trigger();
+  const int G = p.G, H = p.H;
+  const int64_t hrow0 = (int64_t)b * H + g * G;
+  const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
   unsigned err = 0;
-  __syncthreads();
 
-  for (int jt = j0; jt < j1; jt += kGatherTile) {
-    const int n = min(kGatherTile, j1 - jt);
-    // A. stage indices, V rows and logits
-    for (int t = tid; t < kGatherTile; t += kThreads) {
-      const T* vr = nullptr;
-      int i = -1;
-      if (t < n) {
-        i = kept[jt + t];
-        if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
-        else {
-          vr = kv_row<T>(p.v, p, b, g, sq.vs + i);
-          if (!vr) err |= ERR_PAGE;
+  // (a) kept chunk c
+  if (c < p.nk) {
+    const Seq sq = load_seq(p, b, false);
+    const int sel = p.granularity ? b * p.Hkv + g : b;
+    const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
+    const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
+    const int per = (K + p.nk - 1) / p.nk;
+    const int j0 = min(K, c * per), j1 = min(K, j0 + per);
+    if (tid < GM) { sm.run[tid][0] = -CUDART_INF_F; sm.run[tid][1] = 0.f; sm.run[tid][2] = 0.f; }
+    float acc[GM][CH];
+#pragma unroll
+    for (int h = 0; h < GM; ++h)
+#pragma unroll
+      for (int e = 0; e < CH; ++e) acc[h][e] = 0.f;
+    __syncthreads();
+    for (int jt = j0; jt < j1; jt += kGatherTile) {
+      const int n = min(kGatherTile, j1 - jt);
+      if (tid < kGatherTile) {
+        const int t = tid;
+        const T* vr = nullptr;
+        int i = -1;
+        if (t < n) {
+          i = kept[jt + t];
+          if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
+          else {
+            vr = kv_row<T>(p.v, p, b, g, sq.vs + i);
+            if (!vr) err |= ERR_PAGE;
+          }
+        }
+        sm.vrow[t] = vr;
+        const float* zr = p.z_ws + ((int64_t)b * p.max_visual + (i < 0 ? 0 : i)) * p.hp + g * G;
+        float zv[GM];
+#pragma unroll
+        for (int h = 0; h < GM; ++h) zv[h] = (vr && h < G) ? __ldcg(zr + h) : -CUDART_INF_F;
+#pragma unroll
+        for (int h = 0; h < GM; ++h) sm.pz[h][t] = zv[h];
+      }
+      __syncthreads();
+      // per-head tile max and running rescale (warp w handles heads w, w + 8)
+      for (int h = warp; h < G; h += kGatherWarps) {
+        const float z0 = sm.pz[h][lane], z1 = sm.pz[h][lane + 32];
+        const float mo = sm.run[h][0];
+        const float mn = fmaxf(mo, warp_max(fmaxf(z0, z1)));
+        const float e0 = exp2_rel(z0, mn), e1 = exp2_rel(z1, mn);
+        const float ssum = warp_sum(e0 + e1);
+        sm.pz[h][lane] = e0;
+        sm.pz[h][lane + 32] = e1;
+        if (lane == 0) {
+          const float a = exp2_rel(mo, mn);
+          sm.run[h][0] = mn;
+          sm.run[h][1] = sm.run[h][1] * a + ssum;
+          sm.run[h][2] = a;
         }
       }
-      vrow_s[t] = vr;
-      for (int h = 0; h < G; ++h)
-        pz_s[h][t] = vr ? p.z_ws[((int64_t)b * H + g * G + h) * p.max_visual + i] : -CUDART_INF_F;
-    }
-    __syncthreads();
-    // B. per-head tile max and running rescale (warp w handles heads w, w+4, ...)
-    for (int h = warp; h < G; h += kWarps) {
-      const float z0 = pz_s[h][lane], z1 = pz_s[h][lane + 32];
-      const float mt = warp_max(fmaxf(z0, z1));
-      const float mo = run_s[h][0];
-      const float mn = fmaxf(mo, mt);
-      const float e0 = exp2_rel(z0, mn), e1 = exp2_rel(z1, mn);
-      const float ssum = warp_sum(e0 + e1);
-      pz_s[h][lane] = e0;
-      pz_s[h][lane + 32] = e1;
-      if (lane == 0) {
-        const float a = exp2_rel(mo, mn);
-        run_s[h][0] = mn;
-        run_s[h][1] = run_s[h][1] * a + ssum;
-        run_s[h][2] = a;
-      }
-    }
-    __syncthreads();
-    // C. P.V over the staged rows
-#pragma unroll
-    for (int h = 0; h < GM; ++h) {
-      if (h >= G) break;
-      const float a = run_s[h][2];
-#pragma unroll
-      for (int e = 0; e < CH; ++e) acc[h][e] *= a;
-    }
-#pragma unroll 4
-    for (int t = slot; t < n; t += SLOTS) {
-      const T* vr = vrow_s[t];
-      if (!vr) continue;
-      float vv[CH];
-      load_f<CH>(vr + ch * CH, vv);
+      __syncthreads();
 #pragma unroll
       for (int h = 0; h < GM; ++h) {
         if (h >= G) break;
-        const float pr = pz_s[h][t];
+        const float a = sm.run[h][2];
 #pragma unroll
-        for (int e = 0; e < CH; ++e) acc[h][e] = fmaf(pr, vv[e], acc[h][e]);
+        for (int e = 0; e < CH; ++e) acc[h][e] *= a;
+      }
+#pragma unroll 4
+      for (int t = slot; t < n; t += SLOTS) {
+        const T* vr = sm.vrow[t];
+        if (!vr) continue;
+        float vv[CH];
+        load_f<CH>(vr + ch * CH, vv);
+#pragma unroll
+        for (int h = 0; h < GM; ++h) {
+          if (h >= G) break;
+          const float pr = sm.pz[h][t];
+#pragma unroll
+          for (int e = 0; e < CH; ++e) acc[h][e] = fmaf(pr, vv[e], acc[h][e]);
+        }
+      }
+      __syncthreads();
+    }
+    // Reduce the token slots: lanes of one warp first, then a warp tree.
+#pragma unroll
+    for (int o = CPR; o < 32; o <<= 1)
+#pragma unroll
+      for (int h = 0; h < GM; ++h)
+#pragma unroll
+        for (int e = 0; e < CH; ++e) acc[h][e] += __shfl_xor_sync(0xffffffffu, acc[h][e], o);
+    for (int half = kGatherWarps / 2; half >= 1; half >>= 1) {
+      if (warp >= half && warp < 2 * half && lane < CPR) {
+#pragma unroll
+        for (int h = 0; h < GM; ++h)
+#pragma unroll
+          for (int e = 0; e < CH; ++e) sm.red[warp - half][h][ch * CH + e] = acc[h][e];
+      }
+      __syncthreads();
+      if (warp < half && lane < CPR) {
+#pragma unroll
+        for (int h = 0; h < GM; ++h)
+#pragma unroll
+          for (int e = 0; e < CH; ++e) acc[h][e] += sm.red[warp][h][ch * CH + e];
+      }
+      __syncthreads();
+    }
+    if (warp == 0 && lane < CPR) {
+#pragma unroll
+      for (int h = 0; h < GM; ++h) {
+        if (h < G) {
+          float* dst = p.gpart_o + ((pbase + c) * G + h) * D + ch * CH;
+#pragma unroll
+          for (int e = 0; e < CH; ++e) dst[e] = acc[h][e];
+        }
+      }
+    }
+    if (tid < G) {
+      p.gpart_st[((pbase + c) * G + tid) * 2 + 0] = sm.run[tid][0];
+      p.gpart_st[((pbase + c) * G + tid) * 2 + 1] = sm.run[tid][1];
+    }
+  }
+
+  // (b) dimension slice c of the text partials
+  if (c < p.nm) {
+    const int ns = p.ns;
+    for (int i = tid; i < G * ns; i += kGatherThreads) {
+      const int h = i / ns, s = i % ns;
+      const float2 r = __ldcg(reinterpret_cast<const float2*>(p.split_st + ((hrow0 + h) * p.nsp_max + s) * ST_N));
+      sm.tw[h][s] = r.x;  // ST_MT
+      sm.tl[h][s] = r.y;  // ST_L1T
+    }
+    __syncthreads();
+    if (tid < G) {
+      const int h = tid;
+      float M = -CUDART_INF_F;
+      for (int s = 0; s < ns; ++s) M = fmaxf(M, sm.tw[h][s]);
+      float L = 0.f;
+      for (int s = 0; s < ns; ++s) {
+        const float w = exp2_rel(sm.tw[h][s], M);
+        sm.tw[h][s] = w;
+        L = fmaf(w, sm.tl[h][s], L);
+      }
+      if (c == 0) {
+        p.mt_st[(hrow0 + h) * 2 + 0] = M;
+        p.mt_st[(hrow0 + h) * 2 + 1] = L;
       }
     }
     __syncthreads();
+    const int s4 = D4 / p.nm;  // float4s of this CTA's slice, per head
+    for (int i = tid; i < G * s4; i += kGatherThreads) {
+      const int h = i / s4, d = 4 * (c * s4 + i % s4);
+      const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
+      float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+      for (int s = 0; s < ns; ++s) {
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
+        const float w = sm.tw[h][s];
+        num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
+      }
+      *reinterpret_cast<float4*>(p.mt_o + (hrow0 + h) * D + d) = num;
+    }
   }
   if (err) atomicOr(p.err, err);
 
-  // Reduce the token slots (fixed order) and publish this chunk's partial.
-  for (int sl = 0; sl < SLOTS; ++sl) {
-    if (slot == sl) {
-#pragma unroll
-      for (int h = 0; h < GM; ++h) {
-        if (h >= G) break;
-#pragma unroll
-        for (int e = 0; e < CH; ++e) {
-          const float prev = sl == 0 ? 0.f : o_s[h][ch * CH + e];
-          o_s[h][ch * CH + e] = prev + acc[h][e];
-        }
-      }
-    }
-    __syncthreads();
-  }
-  const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
-  for (int i = tid; i < G * D; i += kThreads)
-    p.gpart_o[(pbase + c) * G * D + i] = o_s[i / D][i % D];
-  if (tid < G) {
-    p.gpart_st[((pbase + c) * G + tid) * 2 + 0] = run_s[tid][0];
-    p.gpart_st[((pbase + c) * G + tid) * 2 + 1] = run_s[tid][1];
-  }
   __threadfence();
   __syncthreads();
-  if (tid == 0) {
-    const unsigned t = atomicAdd(p.tickets + (int64_t)b * p.Hkv + g, 1u);
-    last_s = t == (unsigned)p.nk - 1u;
-  }
+  if (tid == 0) sm.last = atomicAdd(p.tickets + (int64_t)b * p.Hkv + g, 1u) == (unsigned)p.nc - 1u;
   __syncthreads();
-  if (!last_s) return;
+  if (!sm.last) return;
   __threadfence();
 
-  // Last chunk: merge text splits and kept chunks in log-sum-exp form.
+  // Last CTA: combine the text output with the kept chunks (log-sum-exp form).
+  // The text part is the merged slice output, or the single split partial.
+  const float* t_o = p.nm ? p.mt_o + hrow0 * D : p.split_o + hrow0 * p.nsp_max * D;
+  const int t_ostride = p.nm ? D : p.nsp_max * D;
   if (tid < G) {
     const int h = tid;
-    float M = -CUDART_INF_F;
-    const float* st = p.split_st + ((int64_t)b * H + g * G + h) * p.ns_max * ST_N;
-    for (int s = 0; s < p.ns; ++s) M = fmaxf(M, st[s * ST_N + ST_MT]);
+    float mt, lt;
+    if (p.nm) {
+      mt = __ldcg(p.mt_st + (hrow0 + h) * 2);
+      lt = __ldcg(p.mt_st + (hrow0 + h) * 2 + 1);
+    } else {
+      mt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_MT);
+      lt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_L1T);
+    }
+    float M = mt;
     for (int k = 0; k < p.nk; ++k) M = fmaxf(M, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2));
-    fin_s[h] = M;
+    const float wt = exp2_rel(mt, M);
+    float den = wt * lt;
+    for (int k = 0; k < p.nk; ++k) {
+      const float w = exp2_rel(__ldcg(p.gpart_st + ((pbase + k) * G + h) * 2), M);
+      sm.tw[h][k] = w;
+      den = fmaf(w, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2 + 1), den);
+    }
+    sm.fin[h][0] = wt;
+    sm.fin[h][1] = den > 0.f ? 1.f / den : 0.f;
   }
   __syncthreads();
-  for (int i = tid; i < G * D; i += kThreads) {
-    const int h = i / D, d = i % D;
-    const float M = fin_s[h];
-    const int64_t hrow = (int64_t)b * H + g * G + h;
-    const float* st = p.split_st + hrow * p.ns_max * ST_N;
-    const float* so = p.split_o + hrow * p.ns_max * D + d;
-    float num = 0.f, den = 0.f;
-    for (int s = 0; s < p.ns; ++s) {
-      const float w = exp2_rel(st[s * ST_N + ST_MT], M);
-      num = fmaf(w, so[(int64_t)s * D], num);
-      den = fmaf(w, st[s * ST_N + ST_L1T], den);
-    }
+  for (int i = tid; i < G * D4; i += kGatherThreads) {
+    const int h = i / D4, d = 4 * (i % D4);
+    const float wt = sm.fin[h][0];
+    const float4 tv = __ldcg(reinterpret_cast<const float4*>(t_o + (int64_t)h * t_ostride + d));
+    float4 num = make_float4(wt * tv.x, wt * tv.y, wt * tv.z, wt * tv.w);
+#pragma unroll 4
     for (int k = 0; k < p.nk; ++k) {
-      const float* gs = p.gpart_st + ((pbase + k) * G + h) * 2;
-      const float w = exp2_rel(__ldcg(gs), M);
-      num = fmaf(w, __ldcg(p.gpart_o + (pbase + k) * G * D + i), num);
-      den = fmaf(w, __ldcg(gs + 1), den);
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(p.gpart_o + ((pbase + k) * G + h) * D + d));
+      const float w = sm.tw[h][k];
+      num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
     }
-    reinterpret_cast<T*>(p.out)[hrow * D + d] = from_f<T>(den > 0.f ? num / den : 0.f);
+    const float inv = sm.fin[h][1];
+    T* o = reinterpret_cast<T*>(p.out) + (hrow0 + h) * D + d;
+    o[0] = from_f<T>(num.x * inv); o[1] = from_f<T>(num.y * inv);
+    o[2] = from_f<T>(num.z * inv); o[3] = from_f<T>(num.w * inv);
   }
   if (tid == 0) p.tickets[(int64_t)b * p.Hkv + g] = 0u;
 }
 
-template <typename T, int D>
-cudaError_t launch_score_td(const StepParams& p, cudaStream_t st) {
-  const dim3 grid(p.ns, p.Hkv, p.B);
-  if (p.G <= 4) k_score<T, D, 4><<<grid, kThreads, 0, st>>>(p);
-  else if (p.G <= 8) k_score<T, D, 8><<<grid, kThreads, 0, st>>>(p);
-  else k_score<T, D, 16><<<grid, kThreads, 0, st>>>(p);
-  return cudaGetLastError();
+// ---------------------------------------------------------------------------
+// k_gather_slice: grid (D / 16, Hkv, B), 256 threads, for kept sets of at most
+// kSliceMaxKept tokens per (sequence, kv-head).  CTA c owns output dimensions
+// [16c, 16c + 16) of the G heads: warps 0-3 attend over every kept visual
+// token (reading only their 16-dimension slice of V), warps 4-7 merge the same
+// slice of the score splits' text partials, and the CTA combines both in
+// log-sum-exp form.  No partial leaves the CTA.
+// ---------------------------------------------------------------------------
+constexpr int kSliceMaxKept = 256;
+constexpr int kSliceDims = 16;
+
+template <int GM>
+struct SliceSmem {
+  int idx[kSliceMaxKept];
+  float pz[GM][kSliceMaxKept];            // kept logits, then probabilities
+  float tm[GM][kNsMax];                   // text split maxima, then weights
+  float tl[GM][kNsMax];                   // text split sums
+  float red[4][GM][kSliceDims];           // kept-part warp partials
+  float4 tred[128];                       // text-part thread partials
+  float fin[GM][4];                       // m_k, l_k, M_t, L_t
+};
+
+template <typename T, int D, int GM>
+__global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_constant__ StepParams p) {
+  constexpr int SD = kSliceDims;
+  constexpr int CH = 16 / sizeof(T);      // elements per 16-byte chunk
+  constexpr int CPS = SD / CH;            // chunks per row slice (2 bf16, 4 fp32)
+  constexpr int TSTRIDE = 128 / CPS;      // kept tokens handled side by side
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  auto& sm = *reinterpret_cast<SliceSmem<GM>*>(smem_raw);
+  const int cd = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  pdl_wait();
+  pdl_trigger();
+  const int G = p.G, H = p.H, ns = p.ns;
+  const int64_t hrow0 = (int64_t)b * H + g * G;
+  const Seq sq = load_seq(p, b, false);
+  const int sel = p.granularity ? b * p.Hkv + g : b;
+  const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, min(p.kept_cap, kSliceMaxKept))));
+  const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
+  unsigned err = 0;
+
+  // 1. Kept indices and their logits; text split statistics (one round trip).
+  for (int t = tid; t < K; t += kGatherThreads) {
+    int i = __ldg(kept + t);
+    if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
+    sm.idx[t] = i;
+    const float* zr = p.z_ws + ((int64_t)b * p.max_visual + (i < 0 ? 0 : i)) * p.hp + g * G;
+    float zv[GM];
+#pragma unroll
+    for (int h = 0; h < GM; ++h) zv[h] = (i >= 0 && h < G) ? __ldcg(zr + h) : -CUDART_INF_F;
+#pragma unroll
+    for (int h = 0; h < GM; ++h) sm.pz[h][t] = zv[h];
+  }
+  for (int i = tid; i < G * ns; i += kGatherThreads) {
+    const int h = i / ns, s = i % ns;
+    const float2 r = __ldcg(reinterpret_cast<const float2*>(p.split_st + ((hrow0 + h) * p.nsp_max + s) * ST_N));
+    sm.tm[h][s] = r.x;  // ST_MT
+    sm.tl[h][s] = r.y;  // ST_L1T
+  }
+  __syncthreads();
+
+  // 2. Per head: kept max / probabilities / sum, text max / weights / sum.
+  for (int h = warp; h < G; h += kGatherWarps) {
+    float m = -CUDART_INF_F;
+    for (int t = lane; t < K; t += 32) m = fmaxf(m, sm.pz[h][t]);
+    m = warp_max(m);
+    float l = 0.f;
+    for (int t = lane; t < K; t += 32) {
+      const float e = exp2_rel(sm.pz[h][t], m);
+      sm.pz[h][t] = e;
+      l += e;
+    }
+    l = warp_sum(l);
+    float mt = -CUDART_INF_F;
+    for (int s = lane; s < ns; s += 32) mt = fmaxf(mt, sm.tm[h][s]);
+    mt = warp_max(mt);
+    float lt = 0.f;
+    for (int s = lane; s < ns; s += 32) {
+      const float w = exp2_rel(sm.tm[h][s], mt);
+      sm.tm[h][s] = w;
+      lt = fmaf(w, sm.tl[h][s], lt);
+    }
+    lt = warp_sum(lt);
+    if (lane == 0) { sm.fin[h][0] = m; sm.fin[h][1] = l; sm.fin[h][2] = mt; sm.fin[h][3] = lt; }
+  }
+  __syncthreads();
+
+  float ko[GM][CH];  // kept part (warps 0-3)
+  if (warp < 4) {
+    // 3a. Kept tokens: thread (token j, chunk q) of the slice.
+    const int j0 = tid / CPS, q = tid % CPS;
+#pragma unroll
+    for (int h = 0; h < GM; ++h)
+#pragma unroll
+      for (int e = 0; e < CH; ++e) ko[h][e] = 0.f;
+#pragma unroll 4
+    for (int j = j0; j < K; j += TSTRIDE) {
+      const int i = sm.idx[j];
+      if (i < 0) continue;
+      const T* vr = kv_row<T>(p.v, p, b, g, sq.vs + i);
+      if (!vr) { err |= ERR_PAGE; continue; }
+      float vv[CH];
+      load_f<CH>(vr + cd * SD + q * CH, vv);
+#pragma unroll
+      for (int h = 0; h < GM; ++h) {
+        if (h >= G) break;
+        const float pr = sm.pz[h][j];
+#pragma unroll
+        for (int e = 0; e < CH; ++e) ko[h][e] = fmaf(pr, vv[e], ko[h][e]);
+      }
+    }
+#pragma unroll
+    for (int o = CPS; o < 32; o <<= 1)
+#pragma unroll
+      for (int h = 0; h < GM; ++h)
+#pragma unroll
+        for (int e = 0; e < CH; ++e) ko[h][e] += __shfl_xor_sync(0xffffffffu, ko[h][e], o);
+    if (lane < CPS) {
+#pragma unroll
+      for (int h = 0; h < GM; ++h)
+#pragma unroll
+        for (int e = 0; e < CH; ++e) sm.red[warp][h][lane * CH + e] = ko[h][e];
+    }
+  } else {
+    // 3b. Text partials: thread (element e = (head, float4), split group sg).
+    const int u = tid - 128;
+    const int NE = G * (SD / 4);
+    const int nsg = 128 / NE;
+    const int e = u % NE, sg = u / NE;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (sg < nsg) {
+      const int h = e / (SD / 4), d = cd * SD + 4 * (e % (SD / 4));
+      const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
+#pragma unroll 4
+      for (int s = sg; s < ns; s += nsg) {
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
+        const float w = sm.tm[h][s];
+        acc.x = fmaf(w, v.x, acc.x); acc.y = fmaf(w, v.y, acc.y); acc.z = fmaf(w, v.z, acc.z); acc.w = fmaf(w, v.w, acc.w);
+      }
+    }
+    sm.tred[u] = acc;
+  }
+  if (err) atomicOr(p.err, err);
+  __syncthreads();
+
+  // 4. Combine (thread per (head, dimension) of the slice).
+  if (tid < G * SD) {
+    const int h = tid / SD, d = tid % SD;
+    float kv = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) kv += sm.red[w][h][d];
+    const int NE = G * (SD / 4), nsg = 128 / NE;
+    const int e = h * (SD / 4) + d / 4;
+    float tv = 0.f;
+    for (int sg = 0; sg < nsg; ++sg) {
+      const float4 v = sm.tred[sg * NE + e];
+      tv += (d & 3) == 0 ? v.x : (d & 3) == 1 ? v.y : (d & 3) == 2 ? v.z : v.w;
+    }
+    const float mk = sm.fin[h][0], lk = sm.fin[h][1], mt = sm.fin[h][2], lt = sm.fin[h][3];
+    const float M = fmaxf(mk, mt);
+    const float ak = exp2_rel(mk, M), at = exp2_rel(mt, M);
+    const float den = ak * lk + at * lt;
+    const float o = den > 0.f ? (ak * kv + at * tv) / den : 0.f;
+    reinterpret_cast<T*>(p.out)[(hrow0 + h) * D + cd * SD + d] = from_f<T>(o);
+  }
 }
+
+// ------------------------------------------------------------------ launching
+
+cudaError_t launch_ex(void (*kernel)(StepParams), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                      int cluster, const StepParams& p) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attrs[2];
+  int na = 0;
+  attrs[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attrs[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (cluster > 1) {
+    attrs[na].id = cudaLaunchAttributeClusterDimension;
+    attrs[na].val.clusterDim.x = cluster;
+    attrs[na].val.clusterDim.y = 1;
+    attrs[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  cfg.attrs = attrs;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, kernel, p);
+}
+
+template <int D, int NT>
+size_t mma_smem() { return MmaCfg<D, NT>::SMEM; }
+template <int D, int GM>
+size_t f32_smem() { return sizeof(F32Smem<D, GM>); }
+template <typename T, int D, int GM>
+size_t gather_smem() { return sizeof(GatherSmem<T, D, GM>); }
+
+template <int D>
+cudaError_t launch_score_d(const StepParams& p, cudaStream_t st) {
+  const dim3 grid(p.ns, p.Hkv, p.B);
+  if (p.dtype == 0) {
+    if (p.G <= 8) return launch_ex(k_score_mma<D, 1>, grid, dim3(kThreads), mma_smem<D, 1>(), st, 1, p);
+    return launch_ex(k_score_mma<D, 2>, grid, dim3(kThreads), mma_smem<D, 2>(), st, 1, p);
+  }
+  if (p.G <= 4) return launch_ex(k_score_f32<D, 4>, grid, dim3(kThreads), f32_smem<D, 4>(), st, 1, p);
+  if (p.G <= 8) return launch_ex(k_score_f32<D, 8>, grid, dim3(kThreads), f32_smem<D, 8>(), st, 1, p);
+  return launch_ex(k_score_f32<D, 16>, grid, dim3(kThreads), f32_smem<D, 16>(), st, 1, p);
+}
+
+template <int GM>
+size_t slice_smem() { return sizeof(SliceSmem<GM>); }
 
 template <typename T, int D>
 cudaError_t launch_gather_td(const StepParams& p, cudaStream_t st) {
-  const dim3 grid(p.nk, p.Hkv, p.B);
-  if (p.G <= 4) k_gather<T, D, 4><<<grid, kThreads, 0, st>>>(p);
-  else if (p.G <= 8) k_gather<T, D, 8><<<grid, kThreads, 0, st>>>(p);
-  else k_gather<T, D, 16><<<grid, kThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  if (p.gslice) {
+    const dim3 grid(D / kSliceDims, p.Hkv, p.B);
+    if (p.G <= 4) return launch_ex(k_gather_slice<T, D, 4>, grid, dim3(kGatherThreads), slice_smem<4>(), st, 1, p);
+    if (p.G <= 8) return launch_ex(k_gather_slice<T, D, 8>, grid, dim3(kGatherThreads), slice_smem<8>(), st, 1, p);
+    return launch_ex(k_gather_slice<T, D, 16>, grid, dim3(kGatherThreads), slice_smem<16>(), st, 1, p);
+  }
+  const dim3 grid(p.nc, p.Hkv, p.B);
+  if (p.G <= 4) return launch_ex(k_gather<T, D, 4>, grid, dim3(kGatherThreads), gather_smem<T, D, 4>(), st, 1, p);
+  if (p.G <= 8) return launch_ex(k_gather<T, D, 8>, grid, dim3(kGatherThreads), gather_smem<T, D, 8>(), st, 1, p);
+  return launch_ex(k_gather<T, D, 16>, grid, dim3(kGatherThreads), gather_smem<T, D, 16>(), st, 1, p);
+}
+
+cudaError_t set_smem(void (*kernel)(StepParams), size_t bytes) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+// The score and gather kernels' shared memory depends only on their template shape.
+cudaError_t configure_fixed_kernels() {
+  cudaError_t e = cudaSuccess;
+#define VP_SET(kernel, bytes) if (e == cudaSuccess) e = set_smem(kernel, bytes)
+  VP_SET((k_score_mma<128, 1>), (mma_smem<128, 1>()));
+  VP_SET((k_score_mma<128, 2>), (mma_smem<128, 2>()));
+  VP_SET((k_score_mma<64, 1>), (mma_smem<64, 1>()));
+  VP_SET((k_score_mma<64, 2>), (mma_smem<64, 2>()));
+  VP_SET((k_score_f32<128, 4>), (f32_smem<128, 4>()));
+  VP_SET((k_score_f32<128, 8>), (f32_smem<128, 8>()));
+  VP_SET((k_score_f32<128, 16>), (f32_smem<128, 16>()));
+  VP_SET((k_score_f32<64, 4>), (f32_smem<64, 4>()));
+  VP_SET((k_score_f32<64, 8>), (f32_smem<64, 8>()));
+  VP_SET((k_score_f32<64, 16>), (f32_smem<64, 16>()));
+  VP_SET((k_gather<__nv_bfloat16, 128, 4>), (gather_smem<__nv_bfloat16, 128, 4>()));
+  VP_SET((k_gather<__nv_bfloat16, 128, 8>), (gather_smem<__nv_bfloat16, 128, 8>()));
+  VP_SET((k_gather<__nv_bfloat16, 128, 16>), (gather_smem<__nv_bfloat16, 128, 16>()));
+  VP_SET((k_gather<__nv_bfloat16, 64, 4>), (gather_smem<__nv_bfloat16, 64, 4>()));
+  VP_SET((k_gather<__nv_bfloat16, 64, 8>), (gather_smem<__nv_bfloat16, 64, 8>()));
+  VP_SET((k_gather<__nv_bfloat16, 64, 16>), (gather_smem<__nv_bfloat16, 64, 16>()));
+  VP_SET((k_gather<float, 128, 4>), (gather_smem<float, 128, 4>()));
+  VP_SET((k_gather<float, 128, 8>), (gather_smem<float, 128, 8>()));
+  VP_SET((k_gather<float, 128, 16>), (gather_smem<float, 128, 16>()));
+  VP_SET((k_gather<float, 64, 4>), (gather_smem<float, 64, 4>()));
+  VP_SET((k_gather<float, 64, 8>), (gather_smem<float, 64, 8>()));
+  VP_SET((k_gather<float, 64, 16>), (gather_smem<float, 64, 16>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 128, 4>), (slice_smem<4>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 128, 8>), (slice_smem<8>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 128, 16>), (slice_smem<16>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 64, 4>), (slice_smem<4>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 64, 8>), (slice_smem<8>()));
+  VP_SET((k_gather_slice<__nv_bfloat16, 64, 16>), (slice_smem<16>()));
+  VP_SET((k_gather_slice<float, 128, 4>), (slice_smem<4>()));
+  VP_SET((k_gather_slice<float, 128, 8>), (slice_smem<8>()));
+  VP_SET((k_gather_slice<float, 128, 16>), (slice_smem<16>()));
+  VP_SET((k_gather_slice<float, 64, 4>), (slice_smem<4>()));
+  VP_SET((k_gather_slice<float, 64, 8>), (slice_smem<8>()));
+  VP_SET((k_gather_slice<float, 64, 16>), (slice_smem<16>()));
+#undef VP_SET
+  return e;
+}
+
+size_t select_smem_bytes(int max_visual, int H, int ns) {
+  return ((size_t)(max_visual > 0 ? max_visual : 1) + 3) / 4 * 16 + (size_t)H * ns * ST_N * sizeof(float);
 }
 
 }  // namespace
 
 cudaError_t launch_score(const StepParams& p, cudaStream_t st) {
-  if (p.dtype == 0)
-    return p.D == 128 ? launch_score_td<__nv_bfloat16, 128>(p, st) : launch_score_td<__nv_bfloat16, 64>(p, st);
-  return p.D == 128 ? launch_score_td<float, 128>(p, st) : launch_score_td<float, 64>(p, st);
+  return p.D == 128 ? launch_score_d<128>(p, st) : launch_score_d<64>(p, st);
 }
 
 cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
@@ -747,26 +1570,18 @@ cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
   return p.D == 128 ? launch_gather_td<float, 128>(p, st) : launch_gather_td<float, 64>(p, st);
 }
 
-size_t select_smem_bytes(int max_visual) { return (size_t)(max_visual > 0 ? max_visual : 1) * sizeof(uint32_t); }
-
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
-  const dim3 grid(p.granularity ? p.Hkv : 1, p.B);
-  k_select<<<grid, kSelThreads, select_smem_bytes(p.max_visual), st>>>(p);
-  return cudaGetLastError();
+  const dim3 grid(p.cl, p.granularity ? p.Hkv : 1, p.B);
+  return launch_ex(k_select, grid, dim3(kSelThreads), select_smem_bytes(p.max_visual, p.H, p.ns), st, p.cl, p);
 }
 
-cudaError_t configure_kernels(int max_visual) {
-  return cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)select_smem_bytes(max_visual));
-}
-
-cudaError_t raise_select_smem(int max_visual) {
+cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {
   cudaFuncAttributes attr;
   cudaError_t e = cudaFuncGetAttributes(&attr, k_select);
   if (e != cudaSuccess) return e;
-  const int need = (int)select_smem_bytes(max_visual);
-  if (attr.maxDynamicSharedSizeBytes >= need) return cudaSuccess;
-  return cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, need);
+  const int need = (int)select_smem_bytes(max_visual, H, nsp_max);
+  if (attr.maxDynamicSharedSizeBytes < need) e = set_smem(k_select, need);
+  return e == cudaSuccess ? configure_fixed_kernels() : e;
 }
 
 }  // namespace vp

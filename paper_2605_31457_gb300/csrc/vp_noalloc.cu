@@ -43,7 +43,6 @@ vp_status fail(vp_status st, const std::string& msg) {
 }
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
-size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Largest K_t of the budget for n visual tokens (same rule as vp_max_kept).
@@ -132,29 +131,17 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   vp_status st = setup_device(dev, &slot);
   if (st != VP_OK) return st;
 
-  // Scratch layout for this call (same partial formats as a context's workspace).
+  // Scratch layout for this call (the partial formats of a context's workspace).
   const int H = c.num_q_heads, Hkv = c.num_kv_heads, G = H / Hkv, D = c.head_dim;
-  const size_t B = (size_t)batch;
-  const int64_t work_max = (int64_t)c.max_visual + 2LL * c.max_seq;
-  const int ns_max = (int)std::max<int64_t>(1, std::min<int64_t>({256, ceil_div(4LL * slot->num_sms, Hkv), ceil_div(work_max, 32)}));
-  const int nk_max = (int)std::max<int64_t>(1, std::min<int64_t>(64, ceil_div(2LL * slot->num_sms, Hkv)));
-  size_t off = 0;
-  const size_t o_t = off; off = round_up(off + B * Hkv * 4, 256);
-  const size_t o_e = off; off = round_up(off + 4, 256);
-  const size_t zero_bytes = off;  // tickets and error word must start at zero
-  const size_t o_z = off; off = round_up(off + B * H * (size_t)std::max(c.max_visual, 1) * 4, 256);
-  const size_t o_st = off; off = round_up(off + B * H * (size_t)ns_max * vp::ST_N * 4, 256);
-  const size_t o_o = off; off = round_up(off + B * H * (size_t)ns_max * D * 4, 256);
-  const size_t o_go = off; off = round_up(off + B * Hkv * (size_t)nk_max * G * D * 4, 256);
-  const size_t o_gs = off; off = round_up(off + B * Hkv * (size_t)nk_max * G * 2 * 4, 256);
-  if (off > (size_t)VP_NOALLOC_SCRATCH_BYTES)
-    return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: this batch and cfg need " + std::to_string(off) +
+  const vp::WsLayout L = vp::ws_layout(batch, H, Hkv, D, c.max_visual, c.max_seq, slot->num_sms);
+  if (L.total > (size_t)VP_NOALLOC_SCRATCH_BYTES)
+    return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: this batch and cfg need " + std::to_string(L.total) +
                 " scratch bytes; the fixed scratch holds " + std::to_string((size_t)VP_NOALLOC_SCRATCH_BYTES));
 
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   char* base = static_cast<char*>(slot->scratch);
-  e = cudaMemsetAsync(base, 0, zero_bytes, stream);
-  if (e == cudaSuccess) e = vp::raise_select_smem(c.max_visual);
+  e = cudaMemsetAsync(base, 0, L.zero_bytes, stream);
+  if (e == cudaSuccess) e = vp::configure_kernels(c.max_visual, H, L.nsp_max);
   if (e != cudaSuccess) return fail(VP_ERR_CUDA, std::string("vp_decode_step_noalloc: ") + cudaGetErrorString(e));
 
   vp::StepParams p;
@@ -178,18 +165,20 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   p.ratio_ppm = budget->ratio_ppm; p.fixed_k = budget->fixed_k;
   p.out = out; p.kept_idx = kept_idx; p.kept_cap = kept_cap; p.kept_count = kept_count;
   p.mass = mass; p.mass_stats = mass_stats;
-  p.tickets = reinterpret_cast<unsigned*>(base + o_t);
-  p.err = reinterpret_cast<unsigned*>(base + o_e);
-  p.z_ws = reinterpret_cast<float*>(base + o_z);
-  p.split_st = reinterpret_cast<float*>(base + o_st);
-  p.split_o = reinterpret_cast<float*>(base + o_o);
-  p.gpart_o = reinterpret_cast<float*>(base + o_go);
-  p.gpart_st = reinterpret_cast<float*>(base + o_gs);
-  p.ns_max = ns_max; p.nk_max = nk_max;
-  const int64_t units = (int64_t)batch * Hkv;
-  p.ns = (int)std::max<int64_t>(1, std::min<int64_t>(ns_max, ceil_div(4LL * slot->num_sms, units)));
-  p.nk = (int)std::max<int64_t>(1, std::min<int64_t>({(int64_t)nk_max, ceil_div(2LL * slot->num_sms, units),
-                                                       std::max<int64_t>(1, ceil_div(kept_cap, 16))}));
+  p.tickets = reinterpret_cast<unsigned*>(base + L.o_tickets);
+  p.err = reinterpret_cast<unsigned*>(base + L.o_err);
+  p.z_ws = reinterpret_cast<float*>(base + L.o_z);
+  p.split_st = reinterpret_cast<float*>(base + L.o_st);
+  p.split_o = reinterpret_cast<float*>(base + L.o_o);
+  p.gpart_o = reinterpret_cast<float*>(base + L.o_go);
+  p.gpart_st = reinterpret_cast<float*>(base + L.o_gs);
+  p.mt_o = reinterpret_cast<float*>(base + L.o_mo);
+  p.mt_st = reinterpret_cast<float*>(base + L.o_ms);
+  const vp::Plan pl = vp::make_plan(batch, Hkv, D, slot->num_sms, c.max_visual, c.max_seq, kept_cap,
+                                    budget->granularity);
+  p.hp = L.hp;
+  p.ns = pl.ns; p.nsp_max = L.nsp_max; p.cl = pl.cl;
+  p.nk = pl.nk; p.nk_max = L.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
   e = vp::launch_score(p, stream);
   if (e == cudaSuccess) e = vp::launch_select(p, stream);
   if (e == cudaSuccess) e = vp::launch_gather(p, stream);
