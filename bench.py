@@ -41,8 +41,10 @@ FALLBACK_HBM_GBS = 6800.0
 def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--steps", type=int, default=None, help="timed steps (default: the workload's)")
     ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--workload", default="qwen7b",
+                    help="qwen7b (default) | serving | long | sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU-baseline leg")
@@ -221,17 +223,46 @@ def run_reference(args, rank, world):
     return 0
 
 
-def workload_config(r):
+def workload_config(r, nbuf=None):
+    import numpy as np
+    bd = r.budget
+    if bd.get("mode", 0) == 0:
+        btxt = f"adaptive tau={bd['tau']} clamp [{bd['r_lo_ppm'] / 1e4:g}%, {bd['r_hi_ppm'] / 1e4:g}%]"
+    else:
+        btxt = f"fixed ratio {bd['ratio_ppm'] / 1e4:g}%"
+    tl = r.text_lens
+    text = f"{int(tl[0])}" if len(set(tl.tolist())) == 1 else f"{int(tl.min())}-{int(tl.max())}"
+    layout = f", paged (page {r.page_size})" if r.paged else ""
+    nb = r.layers if nbuf is None else nbuf
+    step_bytes = r.layers * r.batch * r.kv_heads * r.head_dim * (2 if r.dtype == "bf16" else 4) * \
+        float(np.mean(r.vis_lens + 2 * r.text_lens))
     return {"workload": (f"{r.name}: {r.layers} layers x {r.heads} q / {r.kv_heads} kv heads, "
-                         f"head_dim {r.head_dim}, {r.dtype}, batch {r.batch}, "
-                         f"{int(r.vis_lens[0])} visual + {int(r.text_lens[0])} text tokens at step 0 "
-                         f"(+1 text token per step), budget tau={r.budget['tau']} clamp "
-                         f"[{r.budget['r_lo_ppm'] / 1e4:g}%, {r.budget['r_hi_ppm'] / 1e4:g}%]"),
-            "global_batch": r.batch, "layers": r.layers,
-            "l2": "no flush: each step streams ~0.18 GB of K/V over 28 layers, above the 129 MB L2"}
+                         f"head_dim {r.head_dim}, {r.dtype}{layout}, batch {r.batch}, "
+                         f"{int(r.vis_lens[0])} visual + {text} text tokens at step 0 "
+                         f"(+1 text token per step), budget {btxt}"),
+            "global_batch": r.batch, "layers": r.layers, "distinct_layer_caches": nb,
+            "l2": f"no flush: each step streams ~{step_bytes / 1e9:.2f} GB of K/V; every layer call's "
+                  f"cache is distinct from the previous one's and the per-step stream exceeds the 129 MB L2"}
 
 
 # ------------------------------------------------------------------------ our arm
+
+def pick_workload(name):
+    """(recipe, default timed steps, distinct layer caches, host-generated)."""
+    from paper_2605_31457_gb300 import workloads as W
+    if name == "qwen7b":
+        return W.QWEN7B, 256, W.QWEN7B.layers, True
+    if name == "serving":
+        return W.SERVING, 64, 4, False
+    if name == "long":
+        return W.LONG, 64, 4, False
+    if name.startswith("sweep-"):
+        _, nv, bname = name.split("-")
+        budgets = {"r1": W.SWEEP_BUDGETS[0], "r5": W.SWEEP_BUDGETS[1], "r20": W.SWEEP_BUDGETS[2],
+                   "r50": W.SWEEP_BUDGETS[3], "adaptive": W.SWEEP_BUDGETS[4]}
+        return W.sweep_recipe(int(nv), budgets[bname]), 16, 1, False
+    raise SystemExit(f"unknown workload {name}")
+
 
 def run_ours(args, rank, world, local):
     import numpy as np
@@ -242,33 +273,61 @@ def run_ours(args, rank, world, local):
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    r = W.QWEN7B
+    r, default_steps, nbuf, host_gen = pick_workload(args.workload)
+    if args.steps is None:
+        args.steps = default_steps
     L, B, H, Hkv, D = r.layers, r.batch, r.heads, r.kv_heads, r.head_dim
     S = args.warmup + args.steps
     t_cap = r.capacity(S + 1)
-    nv0, tl0 = int(r.vis_lens[0]), int(r.text_lens[0])
+    nvs, tls = r.vis_lens.astype(np.int64), r.text_lens.astype(np.int64)
+    nv_max = int(nvs.max())
+    cdt = torch.bfloat16 if r.dtype == W.BF16 else torch.float32
 
-    # Inputs: per-layer caches and per-(step, layer) queries, generated on the host.
-    ks, vs_, qs = [], [], []
-    q_host = torch.empty((S, L, B, H, D), dtype=torch.bfloat16)
+    # Inputs: `nbuf` distinct layer caches (layer l reads cache l % nbuf; every
+    # layer call's working set is far larger than L2) and per-(step, layer)
+    # queries.  The default workload is drawn on the host (the generator the
+    # parity tests use); the large ones on the device, same recipe.
+    ks, vs_ = [], []
+    q_dev = torch.empty((S, L, B, H, D), dtype=cdt, device=dev)
+    focus = []
+    for u in range(nbuf):
+        if host_gen:
+            li = W.make_layer(r, u, t_cap=t_cap)
+            ks.append(W.round_to(li.k, r.dtype).to(dev))
+            vs_.append(W.round_to(li.v, r.dtype).to(dev))
+            focus.append(li)
+        else:
+            k, v, f, sk = W.make_layer_torch(r, u, t_cap, dev)
+            ks.append(k)
+            vs_.append(v)
+            focus.append((f, sk))
     for layer in range(L):
-        li = W.make_layer(r, layer, t_cap=t_cap)
-        q = W.make_queries(r, layer, li, steps=S)
-        ks.append(W.round_to(li.k, r.dtype).to(dev))
-        vs_.append(W.round_to(li.v, r.dtype).to(dev))
-        q_host[:, layer] = W.round_to(q, r.dtype)
-    q_dev = q_host.to(dev)
+        u = layer % nbuf
+        if host_gen:
+            q_dev[:, layer] = W.round_to(W.make_queries(r, layer, focus[u], steps=S), r.dtype).to(dev)
+        else:
+            q_dev[:, layer] = W.make_queries_torch(r, layer, S, focus[u][0], focus[u][1], dev)
+    if r.paged:
+        bt_np, n_pages, max_pages = W.page_table(B, t_cap, r.page_size, r.seed)
+        bt = torch.from_numpy(bt_np).to(dev)
+        ks = [W.scatter_pages(k, bt_np, n_pages, r.page_size) for k in ks]
+        vs_ = [W.scatter_pages(v, bt_np, n_pages, r.page_size) for v in vs_]
+        kc = [vp.kv_paged(k, bt) for k in ks]
+        vc = [vp.kv_paged(v, bt) for v in vs_]
+    else:
+        kc = [vp.kv_contiguous(k) for k in ks]
+        vc = [vp.kv_contiguous(v) for v in vs_]
+    torch.cuda.synchronize()
     vis_start = torch.tensor(r.vis_starts, dtype=torch.int32, device=dev)
     vis_len = torch.tensor(r.vis_lens, dtype=torch.int32, device=dev)
     tl_steps = (torch.tensor(r.text_lens, dtype=torch.int32)[None, :] + torch.arange(S, dtype=torch.int32)[:, None]).to(dev)
     span = vp.span(vis_start, vis_len)
-    kc = [vp.kv_contiguous(k) for k in ks]
-    vc = [vp.kv_contiguous(v) for v in vs_]
     budget = vp.make_budget(**r.budget)
-    cfg = vp.make_config(B, H, Hkv, D, nv0, nv0 + tl0 + S, vp.VP_BF16)
+    cfg = vp.make_config(B, H, Hkv, D, nv_max, int((nvs + tls).max()) + S, 
+                         vp.VP_BF16 if r.dtype == W.BF16 else vp.VP_FP32, int(r.paged), r.page_size)
     ctx = vp.vp_init(cfg)
-    cap = vp.vp_max_kept(budget, nv0)
-    out = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
+    cap = max(1, vp.vp_max_kept(budget, nv_max))
+    out = torch.empty((L, B, H, D), dtype=cdt, device=dev)
     kept = torch.empty((L, B, cap), dtype=torch.int32, device=dev)
     count = torch.zeros((S, L, B), dtype=torch.int32, device=dev)
     mass = torch.empty((L, B, H), dtype=torch.float32, device=dev)
@@ -276,7 +335,7 @@ def run_ours(args, rank, world, local):
 
     def step_calls(s, stream=None):
         for layer in range(L):
-            vp.vp_decode_step(ctx, B, q_dev[s, layer], kc[layer], vc[layer], span, tl_steps[s], budget,
+            vp.vp_decode_step(ctx, B, q_dev[s, layer], kc[layer % nbuf], vc[layer % nbuf], span, tl_steps[s], budget,
                               out[layer], kept[layer], cap, count[s, layer], mass[layer], stats[s, layer],
                               stream=stream)
 
@@ -339,7 +398,7 @@ def run_ours(args, rank, world, local):
     for s in range(args.warmup, S):
         for layer in range(L):
             for b in range(B):
-                a, c = call_bytes(r, nv0, tl0 + s, int(counts[s, layer, b]))
+                a, c = call_bytes(r, int(nvs[b]), int(tls[b]) + s, int(counts[s, layer, b]))
                 score_bytes += a
                 gather_bytes += c
     n_calls = args.steps * L
@@ -352,13 +411,13 @@ def run_ours(args, rank, world, local):
     ms_per_step = elapsed_ms / args.steps
     value = world * args.steps / (elapsed_ms * 1e-3)
     step_gbs = (score_bytes + gather_bytes) / (elapsed_ms * 1e-3) / 1e9
-    kept_frac = float(counts[args.warmup:].mean()) / nv0
+    kept_frac = float(counts[args.warmup:].sum() / (args.steps * L * nvs.sum()))
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": dict(workload_config(r), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
+        "config": dict(workload_config(r, nbuf), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
         "hbm": {"achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
                 "frac_of_nominal_8tbs": step_gbs / NOMINAL_HBM_GBS,
                 "bytes_per_step": (score_bytes + gather_bytes) / args.steps,
@@ -377,9 +436,10 @@ def run_ours(args, rank, world, local):
         "gpu_launches": 3 * n_calls,
         "clocks": clocks,
     }
-    if not args.no_e2e:
-        line["e2e"] = e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, world)
-    if not args.no_cpu_baseline and rank == 0:
+    default = args.workload == "qwen7b"
+    if not args.no_e2e and default:
+        line["e2e"] = e2e_leg(args, r, vp, ctx, dev, q_dev.cpu(), ks, vs_, kc, vc, span, budget, cap, world)
+    if not args.no_cpu_baseline and rank == 0 and default:
         times = oracle_times("QWEN7B", list(range(4)), args.warmup, args.cpu_seconds, 4 * L)
         per_call = sum(times) / len(times)
         line["cpu_baseline"] = {"value": 1.0 / (per_call * L), "unit": UNIT, "cores": 1, "kind": "oracle",

@@ -79,7 +79,7 @@ constexpr int kNkMax = 64;    // kept chunks per (sequence, kv-head)
 constexpr int kNsMax = 256;   // score splits per (sequence, kv-head)
 constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
 
-// Launch plan of one call: about one score CTA per SM when the batch is small,
+// Launch plan of one call: score CTAs sized to the work (see below),
 // select clusters that spread the importance scores of few sequences over
 // several SMs, gather chunks of about 256 kept rows.
 struct Plan {
@@ -90,8 +90,12 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
                       int granularity) {
   const long long units = (long long)batch * Hkv;
   const long long tiles = (max_visual + 15) / 16 + 2LL * ((max_seq + 15) / 16);  // work of the longest sequence
+  // One wave of score CTAs (one per SM) while each CTA's share is small; about
+  // four waves once a CTA would stream more than 128 tiles, so that the last
+  // wave's tail costs little.
   long long ns = (num_sms + units - 1) / units;
-  const long long ns_work = tiles / 8 > 1 ? tiles / 8 : 1;  // keep a few tiles per warp
+  if (tiles / ns > 128) ns = (4LL * num_sms + units - 1) / units;
+  const long long ns_work = tiles / 16 > 1 ? tiles / 16 : 1;  // keep a few tiles per warp
   if (ns > ns_work) ns = ns_work;
   if (ns > kNsMax) ns = kNsMax;
   if (ns < 1) ns = 1;

@@ -36,7 +36,7 @@ namespace cg = cooperative_groups;
 namespace vp {
 namespace {
 
-constexpr int kWarps = 4;                 // warps of a score CTA
+constexpr int kWarps = 8;                 // warps of a score CTA
 constexpr int kThreads = 32 * kWarps;
 constexpr int kStages = 3;                // TMA ring depth per warp
 constexpr int kTile = 16;                 // tokens per tile
@@ -423,6 +423,9 @@ __global__ void __launch_bounds__(kThreads) k_score_mma(const __grid_constant__ 
   bool timed_out = false;
   int consumed = 0;  // tiles whose copies were waited for
   for (int k = 0; k < my_n; ++k) {
+    // Tile k + 2 goes into the stage tile k - 1 used (consumed last iteration),
+    // so all three stages are in flight while this warp waits for tile k.
+    issue(k + kStages - 1);
     if (!mbar_wait(bars + k % kStages, (k / kStages) & 1)) { timed_out = true; break; }
     consumed = k + 1;
     const int j = warp + kWarps * k;
@@ -540,7 +543,6 @@ __global__ void __launch_bounds__(kThreads) k_score_mma(const __grid_constant__ 
       }
     }
     __syncwarp();
-    issue(k + kStages - 1);
   }
   // After a timed-out wait, the copies still in flight must land (or time out
   // again) before the ring is reused for the partials or the CTA exits.

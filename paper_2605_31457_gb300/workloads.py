@@ -251,3 +251,70 @@ SWEEP_BUDGETS = tuple(dict(mode=1, tau=0.1, ratio_ppm=r) for r in (10_000, 50_00
 def shrink(r: Recipe, **kw) -> Recipe:
     """A smaller copy of a recipe (tests)."""
     return replace(r, **kw)
+
+
+# ---------------------------------------------------------------------------
+# The same recipe drawn on the GPU with torch's seeded generator, for the
+# benchmark's large workloads (gigabytes of cache; host generation would take
+# minutes).  Values differ from the host generator's; the recipe is the same.
+# ---------------------------------------------------------------------------
+
+def make_layer_torch(r: Recipe, layer: int, t_cap: int, device, dtype=None):
+    """Keys and values [B, Hkv, t_cap, D] (cache dtype) plus the focus and
+    sink directions [n_focus, B, Hkv, D] / [B, Hkv, D] (float32)."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(r.seed) * 1_000_003 + int(layer) * 7_919 + 11)
+    B, Hkv, D = r.batch, r.kv_heads, r.head_dim
+    dt = dtype or (torch.bfloat16 if r.dtype == BF16 else torch.float32)
+    k = torch.randn((B, Hkv, t_cap, D), generator=gen, device=device, dtype=torch.float32)
+    v = torch.randn((B, Hkv, t_cap, D), generator=gen, device=device, dtype=torch.float32).to(dt)
+    focus = torch.randn((r.n_focus, B, Hkv, D), generator=gen, device=device)
+    focus = focus / focus.norm(dim=-1, keepdim=True)
+    sink = torch.randn((B, Hkv, D), generator=gen, device=device)
+    sink = sink - (sink * focus[0]).sum(-1, keepdim=True) * focus[0]
+    sink = sink / sink.norm(dim=-1, keepdim=True)
+    sqd = math.sqrt(D)
+    vs, vl = r.vis_starts, r.vis_lens
+    for f in range(r.n_focus):
+        for b in range(B):
+            nv = int(vl[b])
+            n_p = min(nv, int(round(r.planted_frac * nv)))
+            if not n_p:
+                continue
+            pos = torch.randperm(nv, generator=gen, device=device)[:n_p] + int(vs[b])
+            u = focus[f, b][:, None, :].expand(Hkv, n_p, D)
+            w = torch.randn((Hkv, n_p, D), generator=gen, device=device)
+            w = w - (w * u).sum(-1, keepdim=True) * u
+            w = w / w.norm(dim=-1, keepdim=True)
+            k[b, :, pos, :] = sqd * (0.8 * u + 0.6 * w)
+    if r.beta_sink > 0:
+        for b in range(B):
+            first_text = 0 if vs[b] > 0 else int(vl[b])
+            k[b, :, first_text, :] = sqd * sink[b]
+    if r.key_sigma > 0:
+        k *= torch.exp(r.key_sigma * torch.randn((B, Hkv, t_cap, 1), generator=gen, device=device))
+    return k.to(dt), v, focus, sink
+
+
+def make_queries_torch(r: Recipe, layer: int, steps: int, focus, sink, device, dtype=None):
+    """Queries [steps, B, H, D] in the cache dtype (same recipe as make_queries)."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(r.seed) * 1_000_003 + int(layer) * 7_919 + 23)
+    B, H, Hkv, D = r.batch, r.heads, r.kv_heads, r.head_dim
+    G = H // Hkv
+    lo, hi = r.beta_range
+    beta = torch.exp(math.log(lo) + (math.log(hi) - math.log(lo)) *
+                     torch.rand((steps, B, H), generator=gen, device=device))
+    if r.seq_beta:
+        beta = beta * torch.tensor(r.seq_beta, device=device)[None, :, None]
+    fidx = torch.zeros(steps, dtype=torch.long, device=device)
+    if r.focus_every > 0:
+        fidx = (torch.arange(steps, device=device) // r.focus_every) % r.n_focus
+    u = focus[fidx].repeat_interleave(G, dim=2)                  # [steps, B, H, D]
+    us = sink.repeat_interleave(G, dim=1)[None]
+    noise = torch.randn((steps, B, H, D), generator=gen, device=device)
+    q = math.sqrt(D) * (beta[..., None] * u + r.beta_sink * us) + noise
+    dt = dtype or (torch.bfloat16 if r.dtype == BF16 else torch.float32)
+    return q.to(dt)
