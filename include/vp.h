@@ -76,7 +76,10 @@ typedef struct {
  * (strides in elements; the d axis is contiguous).  Every row (D elements)
  * must start on a 16-byte boundary: data 16-byte aligned and every stride a
  * multiple of 16 bytes.  A page id outside [0, num_pages) is skipped and
- * flagged.
+ * flagged.  The kernels read whole 32-token tiles: in a contiguous cache,
+ * rows t < max_seq of every (sequence, kv-head) must be readable memory, and
+ * in a paged cache every row of a mapped page; rows past the live length are
+ * read but never used.
  */
 typedef struct {
   const void* data;

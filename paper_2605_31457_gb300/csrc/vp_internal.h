@@ -2,8 +2,9 @@
 // (vp_kernels.cu) of libvp.  Not part of the public ABI.
 #pragma once
 
-#include <stdint.h>
+#include <cuda.h>  // CUtensorMap (type only; the library does not link the driver)
 #include <cuda_runtime.h>
+#include <stdint.h>
 
 namespace vp {
 
@@ -31,6 +32,11 @@ struct KvView {
 };
 
 struct StepParams {
+  // bulk-tensor (TMA) descriptors of the K and V caches (bf16), when use_tma
+  CUtensorMap tmk;  // 64-byte aligned type
+  CUtensorMap tmv;
+  int use_tma;
+  int tpos, gpos, bpos;  // descriptor dimension (1..3) of the token, kv-head and sequence/page axes
   // shapes
   int dtype;  // 0 = bf16, 1 = fp32 (vp_dtype)
   int B, H, Hkv, G, D;
@@ -89,16 +95,23 @@ struct Plan {
 inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, int max_seq, int kept_cap,
                       int granularity) {
   const long long units = (long long)batch * Hkv;
-  const long long tiles = (max_visual + 15) / 16 + 2LL * ((max_seq + 15) / 16);  // work of the longest sequence
-  // One wave of score CTAs (one per SM) while each CTA's share is small; about
-  // four waves once a CTA would stream more than 128 tiles, so that the last
-  // wave's tail costs little.
-  long long ns = (num_sms + units - 1) / units;
-  if (tiles / ns > 128) ns = (4LL * num_sms + units - 1) / units;
-  const long long ns_work = tiles / 16 > 1 ? tiles / 16 : 1;  // keep a few tiles per warp
-  if (ns > ns_work) ns = ns_work;
-  if (ns > kNsMax) ns = kNsMax;
-  if (ns < 1) ns = 1;
+  // Work of the longest sequence in 32-token tiles (text tiles carry K and V,
+  // so they weigh 2).  Score CTAs are small enough that two fit on an SM.
+  const long long tiles = (max_visual + 31) / 32 + 2LL * ((max_seq + 31) / 32);
+  const long long slots = 2LL * num_sms;
+  // Split count: minimise (waves of CTAs) x (tiles per CTA + a fixed cost of
+  // about 4 tiles per CTA for its start and its partial), keeping at least 8
+  // tiles per CTA; the smaller count wins a tie.
+  long long ns_hi = tiles / 8;
+  if (ns_hi > kNsMax) ns_hi = kNsMax;
+  if (ns_hi < 1) ns_hi = 1;
+  long long ns = 1;
+  double best = 0.0;
+  for (long long c = 1; c <= ns_hi; ++c) {
+    const double waves = (double)((units * c + slots - 1) / slots);
+    const double cost = waves * ((double)tiles / (double)c + 4.0);
+    if (c == 1 || cost < best * (1.0 - 1e-9)) { best = cost; ns = c; }
+  }
   const long long sel = (long long)batch * (granularity ? Hkv : 1);
   int cl = 1;
   while (cl < 8 && sel * cl * 2 <= num_sms) cl *= 2;
@@ -150,5 +163,9 @@ cudaError_t launch_gather(const StepParams& p, cudaStream_t s);
 // Kernel attributes: raises (never lowers) the select kernel's dynamic
 // shared-memory limit for these shapes and sets the other kernels' limits.
 cudaError_t configure_kernels(int max_visual, int H, int nsp_max);
+// Fills p.tmk / p.tmv / p.use_tma for a bf16 cache whose layout a 4-D tensor
+// descriptor can describe without reaching past the caller's memory; leaves
+// use_tma = 0 otherwise (the score kernel then copies rows one by one).
+void encode_kv_maps(StepParams& p);
 
 }  // namespace vp

@@ -45,7 +45,7 @@ constexpr int kMaxHeads = 128;
 constexpr int kGatherThreads = 256;
 constexpr int kGatherWarps = kGatherThreads / 32;
 constexpr int kGatherTile = 64;           // kept tokens staged per round in k_gather
-constexpr long long kSpinLimit = 1LL << 22;  // mbarrier polls before a wait gives up
+constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // an mbarrier wait gives up after 1 s
 
 // Budget modes (numbering of vp_budget_mode in include/vp.h).
 enum { MODE_ADAPTIVE = 0, MODE_FIXED_RATIO = 1, MODE_FIXED_K = 2, MODE_DENSE = 3 };
@@ -170,13 +170,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
       : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
   return ok != 0;
 }
-// Bounded wait for a phase of an mbarrier; false if it never completed.
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait for a phase of an mbarrier; false if it did not complete
+// within kWaitLimitNs.  try_wait itself suspends the thread until the phase
+// completes or a hardware time slice ends, so the loop needs no sleep.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
-  for (long long i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (i > 32) __nanosleep(64);
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (;;) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > kWaitLimitNs) return false;
   }
-  return false;
 }
 // Orders this thread's earlier generic-proxy shared-memory accesses before
 // later asynchronous-proxy (bulk copy) writes to the same memory.
@@ -260,29 +269,30 @@ __device__ __forceinline__ void merge_stats(const float* recs, int n, int stride
 }
 
 // ------------------------------------------------------- score epilogue
-// Shared by both score kernels: per-warp statistics wst[w][h][ST_N] and text
+// Shared by the score kernels: per-warp statistics wst[w][h][ST_N] and text
 // outputs (warp w at ow + w * ow_stride, [GM][D]) are merged into the CTA's
 // partial and written to split slot s.
-template <int GM, int D>
+template <int GM, int D, int NW = kWarps>
 struct ScoreTail {
   float cst[GM][ST_N];
-  float wsc[kWarps][GM];
+  float wsc[NW][GM];
 };
 
-template <int GM, int D>
+// NW warp records are merged; the kernel runs NTHR threads.
+template <int GM, int D, int NW = kWarps, int NTHR = kThreads>
 __device__ void score_epilogue(const StepParams& p, int b, int g, int s, const float (*wst)[GM][ST_N],
-                               const float* ow, int ow_stride, ScoreTail<GM, D>& tl) {
+                               const float* ow, int ow_stride, ScoreTail<GM, D, NW>& tl) {
   const int tid = threadIdx.x, G = p.G;
   constexpr int D4 = D / 4;
   __syncthreads();
-  if (tid < G) merge_stats(&wst[0][tid][0], kWarps, GM * ST_N, p.inv_tau, tl.cst[tid], &tl.wsc[0][tid], GM);
+  if (tid < G) merge_stats(&wst[0][tid][0], NW, GM * ST_N, p.inv_tau, tl.cst[tid], &tl.wsc[0][tid], GM);
   __syncthreads();
   const int64_t rec0 = ((int64_t)b * p.H + g * G) * p.nsp_max + s;  // slot of head 0
-  for (int i = tid; i < G * D4; i += kThreads) {
+  for (int i = tid; i < G * D4; i += NTHR) {
     const int h = i / D4, d = 4 * (i % D4);
     float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
+    for (int w = 0; w < NW; ++w) {
       const float a = tl.wsc[w][h];
       const float4 v = *reinterpret_cast<const float4*>(ow + w * ow_stride + h * D + d);
       o.x = fmaf(a, v.x, o.x); o.y = fmaf(a, v.y, o.y); o.z = fmaf(a, v.z, o.z); o.w = fmaf(a, v.w, o.w);
@@ -579,6 +589,428 @@ __global__ void __launch_bounds__(kThreads) k_score_mma(const __grid_constant__ 
       ow[(h0 + 1) * D + d0 + 8] = acc[n][mi][3];
     }
   score_epilogue<GM, D>(p, b, g, s, wst, reinterpret_cast<const float*>(smem), C::RING / 4, tail);
+}
+
+// ---------------------------------------------------------------------------
+// k_score_tma (bf16).  The CTA's token range is cut into 32-token tiles
+// aligned to absolute cache positions; warp w takes tiles w, w + NW, ...
+// Every warp streams its own tiles through a private ring of S tile-sized
+// slots in shared memory: lane 0 arms a slot's mbarrier with its byte count
+// and loads the tile with 4-D bulk-tensor (TMA) copies -- boxes of 64
+// dimensions x 32 rows (fewer when a page is shorter) with the 128-byte
+// hardware swizzle, so the ldmatrix reads below are free of bank conflicts.
+// A tile wholly inside the visual span takes one slot (K only); any other
+// tile takes two consecutive slots (K, then V).  A warp refills a slot as soon
+// as it has read it (K right after QK, V after PV), so up to S slots of its
+// tiles are in flight.  Because each warp waits on its own slots strictly in
+// the order it armed them, a barrier is never waited on more than one phase
+// ahead.  QK and PV run on the tensor cores as in k_score_mma.  Rows past the
+// live cache, or of an unmapped page, are masked by a row mask stored with
+// the slot.  For paged caches the page ids of the CTA's boxes are read into
+// shared memory once, before the first copy.
+// ---------------------------------------------------------------------------
+constexpr int kTmaTile = 32;
+constexpr int kTmaMaxBoxes = 1024;  // page-id entries per cache a CTA may hold
+
+template <int D, int NT, int NW, int S>
+struct TmaCfg {
+  static constexpr int GM = 8 * NT;
+  static constexpr int THREADS = 32 * NW;
+  static constexpr int KS = D / 16;                      // QK k-steps
+  static constexpr int MT = D / 16;                      // PV m-tiles
+  static constexpr int HALVES = D / 64;                  // 64-dimension boxes per row
+  static constexpr int HALF_BYTES = kTmaTile * 128;      // one box: 32 rows x 128 bytes
+  static constexpr int SLOT = HALVES * HALF_BYTES;       // one tile of K or of V
+  static constexpr int RING = NW * S * SLOT;
+  static constexpr int OFF_BAR = RING;                   // full[NW][S]
+  static constexpr int OFF_MASK = OFF_BAR + NW * S * 8;  // row mask per slot
+  static constexpr int OFF_PG = (OFF_MASK + NW * S * 4 + 15) / 16 * 16;  // page ids, K then V
+  static constexpr int OFF_TAIL = OFF_PG + 2 * kTmaMaxBoxes * 4;
+  static constexpr int OFF_WST = OFF_TAIL + (int)sizeof(ScoreTail<GM, D, NW>);
+  static constexpr size_t SMEM = 1024 + (size_t)OFF_WST + sizeof(float) * NW * GM * ST_N;
+  static_assert(S >= 2, "a text tile needs two slots");
+  static_assert(NW * GM * D * 4 <= RING, "text partials must fit in the ring");
+  static_assert(SLOT % 1024 == 0, "slots keep the swizzle atoms aligned");
+};
+
+// Byte offset of (row, element col) in a swizzled tile of 64-element boxes.
+template <int HALF_BYTES>
+__device__ __forceinline__ unsigned swz_off(int row, int col) {
+  return (unsigned)((col >> 6) * HALF_BYTES + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4));
+}
+__device__ __forceinline__ float fexp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ void tma_load_4d(unsigned dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];\n"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Page of the pool that holds cache position pos of sequence b; -1 if the
+// block table maps it nowhere.
+__device__ __forceinline__ int tma_page(const KvView& kv, const StepParams& p, int b, int pos) {
+  const int lp = pos >> p.page_shift;
+  if (lp >= kv.max_pages) return -1;
+  const int page = __ldg(kv.block_table + (int64_t)b * kv.max_pages + lp);
+  return (page < 0 || page >= kv.num_pages) ? -1 : page;
+}
+
+// The tiles of one split.  Tiles [v0, v1) lie wholly inside the visual span
+// (K only); every other tile carries text rows (K and V).  Split s owns
+// tiles [u0, u0 + n), cut so that every split moves about the same bytes.
+struct TileRange {
+  int u0, n, v0, v1;
+  __device__ __forceinline__ bool text(int t) const {
+    const int u = u0 + t;
+    return u < v0 || u >= v1;
+  }
+};
+__device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns) {
+  const int T = sq.nv + sq.tl;
+  const int NTl = (T + kTmaTile - 1) / kTmaTile;
+  const int v0 = (sq.vs + kTmaTile - 1) / kTmaTile;
+  const int v1 = max(v0, min(NTl, (sq.vs + sq.nv) / kTmaTile));
+  const int W = 2 * NTl - (v1 - v0);  // text tiles weigh 2, visual tiles 1
+  const int per = (W + ns - 1) / ns;
+  auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
+    if (w <= 2 * v0) return (w + 1) / 2;
+    if (w <= v0 + v1) return w - v0;
+    return (w + (v1 - v0) + 1) / 2;
+  };
+  TileRange r;
+  r.u0 = tile_of(min(W, s * per));
+  r.n = tile_of(min(W, (s + 1) * per)) - r.u0;
+  r.v0 = v0;
+  r.v1 = v1;
+  return r;
+}
+
+template <int D, int NT, int NW, int S>
+__global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant__ StepParams p) {
+  using C = TmaCfg<D, NT, NW, S>;
+  constexpr int GM = C::GM;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  // The 128-byte swizzle repeats every 1024 bytes: align the ring to that.
+  unsigned char* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gr = lane >> 2, tg = lane & 3;
+  const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + warp * S;
+  uint32_t* rowmask = reinterpret_cast<uint32_t*>(smem + C::OFF_MASK) + warp * S;
+  int* kpg = reinterpret_cast<int*>(smem + C::OFF_PG);
+  int* vpg = kpg + kTmaMaxBoxes;
+  unsigned char* ring = smem + warp * S * C::SLOT;
+  auto& tail = *reinterpret_cast<ScoreTail<GM, D, NW>*>(smem + C::OFF_TAIL);
+  auto wst = reinterpret_cast<float (*)[GM][ST_N]>(smem + C::OFF_WST);
+
+  if (tid < NW * S) mbar_init(reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + tid, 1);
+  mbar_fence_init();
+  pdl_wait();
+  const int G = p.G, H = p.H;
+  const Seq sq = load_seq(p, b, s == 0 && g == 0);
+  const int T = sq.nv + sq.tl;
+  const TileRange tr = tma_split(sq, s, p.ns);
+  const int R = p.paged ? min(kTmaTile, p.page_size) : kTmaTile;  // rows per box
+  const int nb = kTmaTile / R;                                     // boxes per tile (1..4)
+  int n = tr.n;
+  unsigned err = 0;
+  if (p.paged) {
+    if (n * nb > kTmaMaxBoxes) {  // the host plan keeps every CTA below this
+      err |= ERR_PAGE;
+      n = 0;
+    }
+    for (int i = tid; i < n * nb; i += C::THREADS) {
+      const int t = i / nb, pos = (tr.u0 + t) * kTmaTile + (i % nb) * R;
+      kpg[i] = pos < T ? tma_page(p.k, p, b, pos) : -2;
+      vpg[i] = (pos < T && tr.text(t)) ? tma_page(p.v, p, b, pos) : 0;
+    }
+  }
+  __syncthreads();
+
+  // ---------------------------------------------------------------- issue
+  const int nj = warp < n ? (n - warp + NW - 1) / NW : 0;  // this warp's tiles
+  int ji = 0, qi = 0, qf = 0;  // next tile to issue, its first slot, first slot not yet read
+  const uint32_t boxmask = R >= 32 ? 0xffffffffu : ((1u << R) - 1u);
+  auto issue = [&]() {
+    while (ji < nj) {
+      const int t = warp + NW * ji;
+      const bool text = tr.text(t);
+      const int need = text ? 2 : 1;
+      if (qi + need - qf > S) break;
+      // The slots were last read by this warp's ldmatrix (generic proxy).
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) {
+        const int p0 = (tr.u0 + t) * kTmaTile;
+        const int nvalid = min(kTmaTile, T - p0);
+        uint32_t mask = nvalid >= 32 ? 0xffffffffu : ((1u << nvalid) - 1u);
+        const int ks = qi % S, vs = (qi + 1) % S;
+        unsigned bytes = 0;
+        int kb[4], vb[4];
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+          kb[x] = -1;
+          vb[x] = 0;
+          if (x < nb && p0 + x * R < T) {
+            if (p.paged) {
+              kb[x] = kpg[t * nb + x];
+              vb[x] = vpg[t * nb + x];
+            } else {
+              kb[x] = vb[x] = b;
+            }
+            if (kb[x] < 0 || vb[x] < 0) {
+              err |= ERR_PAGE;
+              mask &= ~(boxmask << (x * R));
+              kb[x] = -1;
+            } else {
+              bytes += C::HALVES * R * 128u;
+            }
+          }
+        }
+        rowmask[ks] = mask;
+        mbar_expect_tx(full + ks, bytes);
+        if (text) mbar_expect_tx(full + vs, bytes);
+        const unsigned kt = smem_u32(ring + ks * C::SLOT), vt = smem_u32(ring + vs * C::SLOT);
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+          if (kb[x] < 0) continue;
+          const int row = p.paged ? ((p0 + x * R) & (p.page_size - 1)) : p0 + x * R;
+          auto crd = [&](int axis, int base) { return axis == p.tpos ? row : axis == p.gpos ? g : base; };
+#pragma unroll
+          for (int hh = 0; hh < C::HALVES; ++hh) {
+            const unsigned off = hh * C::HALF_BYTES + x * R * 128;
+            tma_load_4d(kt + off, &p.tmk, 64 * hh, crd(1, kb[x]), crd(2, kb[x]), crd(3, kb[x]), full + ks);
+            if (text) tma_load_4d(vt + off, &p.tmv, 64 * hh, crd(1, vb[x]), crd(2, vb[x]), crd(3, vb[x]), full + vs);
+          }
+        }
+      }
+      qi += need;
+      ++ji;
+    }
+  };
+  issue();
+
+  // -------------------------------------------------------------- consume
+  uint32_t qfr[NT][C::KS][2];
+  const __nv_bfloat16* qb = reinterpret_cast<const __nv_bfloat16*>(p.q) + ((int64_t)b * H + g * G) * D;
+#pragma unroll
+  for (int nn = 0; nn < NT; ++nn) {
+    const int h = 8 * nn + gr;
+    const uint32_t* qr = reinterpret_cast<const uint32_t*>(qb + h * D);
+#pragma unroll
+    for (int ks = 0; ks < C::KS; ++ks) {
+      qfr[nn][ks][0] = h < G ? __ldg(qr + 8 * ks + tg) : 0u;
+      qfr[nn][ks][1] = h < G ? __ldg(qr + 8 * ks + 4 + tg) : 0u;
+    }
+  }
+  float m_v[NT][2], l1v[NT][2], ltv[NT][2], m_t[NT][2], l1t[NT][2], ltt[NT][2];
+  float acc[NT][C::MT][4];
+#pragma unroll
+  for (int nn = 0; nn < NT; ++nn) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      m_v[nn][j] = m_t[nn][j] = -CUDART_INF_F;
+      l1v[nn][j] = ltv[nn][j] = l1t[nn][j] = ltt[nn][j] = 0.f;
+    }
+#pragma unroll
+    for (int mi = 0; mi < C::MT; ++mi)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[nn][mi][e] = 0.f;
+  }
+  // ldmatrix lane roles: K as the A operand (rows = tokens), V^T via .trans.
+  const int krow = (lane & 7) + 8 * ((lane >> 3) & 1), kcol = 8 * (lane >> 4);
+  const int vrow = (lane & 7) + 8 * (lane >> 4), vcol = 8 * ((lane >> 3) & 1);
+  const float ctau = p.inv_tau;
+  bool timed_out = false;
+  int qc = 0;  // first slot of the tile being read
+
+  for (int j = 0; j < nj; ++j) {
+    const int t = warp + NW * j;
+    const bool text = tr.text(t);
+    const int ks_ = qc % S;
+    if (!mbar_wait(full + ks_, (qc / S) & 1)) { timed_out = true; break; }
+    const uint32_t mask = rowmask[ks_];
+    const int p0 = (tr.u0 + t) * kTmaTile;
+    const unsigned kt = smem_u32(ring + ks_ * C::SLOT);
+
+    // ---- QK for both 16-row halves of the tile, then refill the K slot
+    float c[2][NT][4];
+#pragma unroll
+    for (int sb = 0; sb < 2; ++sb) {
+#pragma unroll
+      for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) c[sb][nn][e] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < C::KS; ++ks) {
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(kt + swz_off<C::HALF_BYTES>(16 * sb + krow, 16 * ks + kcol), a0, a1, a2, a3);
+#pragma unroll
+        for (int nn = 0; nn < NT; ++nn) mma_bf16(c[sb][nn], a0, a1, a2, a3, qfr[nn][ks][0], qfr[nn][ks][1]);
+      }
+    }
+    qf = qc + 1;
+    issue();
+
+    // c[sb][n][e]: row 16sb + gr + 8(e >> 1), head 8n + 2tg + (e & 1).
+    float zv[2][NT][4], zt[2][NT][4];
+    bool any_vis = false;
+#pragma unroll
+    for (int sb = 0; sb < 2; ++sb)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int row = 16 * sb + gr + 8 * (e >> 1);
+        const int pos = p0 + row;
+        const bool valid = (mask >> row) & 1u;
+        const bool vis = valid && (unsigned)(pos - sq.vs) < (unsigned)sq.nv;
+        any_vis |= vis;
+#pragma unroll
+        for (int nn = 0; nn < NT; ++nn) {
+          const bool hv = (8 * nn + 2 * tg + (e & 1)) < G;
+          const float z = c[sb][nn][e] * p.c_log2;
+          zv[sb][nn][e] = (vis && hv) ? z : -CUDART_INF_F;
+          zt[sb][nn][e] = (valid && !vis && hv) ? z : -CUDART_INF_F;
+        }
+        if (vis) {
+          float* zrow = p.z_ws + ((int64_t)b * p.max_visual + (pos - sq.vs)) * p.hp + g * G;
+#pragma unroll
+          for (int nn = 0; nn < NT; ++nn) {
+            const int h = 8 * nn + 2 * tg + (e & 1);
+            if (h < G) zrow[h] = zv[sb][nn][e];
+          }
+        }
+      }
+    // ---- visual statistics
+    if (__any_sync(0xffffffffu, any_vis)) {
+#pragma unroll
+      for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          const float mx = fmaxf(fmaxf(zv[0][nn][jj], zv[0][nn][jj + 2]), fmaxf(zv[1][nn][jj], zv[1][nn][jj + 2]));
+          const float mn = fmaxf(m_v[nn][jj], group_max(mx));
+          if (mn > m_v[nn][jj]) {
+            l1v[nn][jj] *= exp2_rel(m_v[nn][jj], mn);
+            ltv[nn][jj] *= exp2_tau(m_v[nn][jj], mn, ctau);
+            m_v[nn][jj] = mn;
+          }
+          if (mn != -CUDART_INF_F) {
+#pragma unroll
+            for (int sb = 0; sb < 2; ++sb)
+#pragma unroll
+              for (int e = jj; e < 4; e += 2) {
+                l1v[nn][jj] += fexp2(zv[sb][nn][e] - mn);
+                ltv[nn][jj] += fexp2((zv[sb][nn][e] - mn) * ctau);
+              }
+          }
+        }
+    }
+    // ---- text statistics, probabilities and P.V from the V slot
+    if (text) {
+      uint32_t pb[2][NT][2];
+#pragma unroll
+      for (int nn = 0; nn < NT; ++nn) {
+        float pr[2][4];
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          const float mx = fmaxf(fmaxf(zt[0][nn][jj], zt[0][nn][jj + 2]), fmaxf(zt[1][nn][jj], zt[1][nn][jj + 2]));
+          const float mn = fmaxf(m_t[nn][jj], group_max(mx));
+          if (mn > m_t[nn][jj]) {
+            const float a = exp2_rel(m_t[nn][jj], mn);
+            l1t[nn][jj] *= a;
+            ltt[nn][jj] *= exp2_tau(m_t[nn][jj], mn, ctau);
+#pragma unroll
+            for (int mi = 0; mi < C::MT; ++mi) {
+              acc[nn][mi][jj] *= a;
+              acc[nn][mi][jj + 2] *= a;
+            }
+            m_t[nn][jj] = mn;
+          }
+#pragma unroll
+          for (int sb = 0; sb < 2; ++sb)
+#pragma unroll
+            for (int e = jj; e < 4; e += 2) {
+              const float pe = mn != -CUDART_INF_F ? fexp2(zt[sb][nn][e] - mn) : 0.f;
+              pr[sb][e] = pe;
+              l1t[nn][jj] += pe;
+              if (mn != -CUDART_INF_F) ltt[nn][jj] += fexp2((zt[sb][nn][e] - mn) * ctau);
+            }
+        }
+#pragma unroll
+        for (int sb = 0; sb < 2; ++sb) {
+          const uint32_t p01 = pack_bf16(pr[sb][0], pr[sb][1]), p23 = pack_bf16(pr[sb][2], pr[sb][3]);
+          const int src0 = 8 * tg + (gr >> 1), src1 = src0 + 4;
+          const uint32_t x0 = __shfl_sync(0xffffffffu, p01, src0), x1 = __shfl_sync(0xffffffffu, p01, src1);
+          const uint32_t x2 = __shfl_sync(0xffffffffu, p23, src0), x3 = __shfl_sync(0xffffffffu, p23, src1);
+          const uint32_t sel = (gr & 1) ? 0x7632u : 0x5410u;
+          pb[sb][nn][0] = prmt(x0, x1, sel);
+          pb[sb][nn][1] = prmt(x2, x3, sel);
+        }
+      }
+      const int vq = qc + 1, vs_ = vq % S;
+      if (!mbar_wait(full + vs_, (vq / S) & 1)) { timed_out = true; break; }
+      const unsigned vt = smem_u32(ring + vs_ * C::SLOT);
+#pragma unroll
+      for (int sb = 0; sb < 2; ++sb) {
+        // Words of rows outside the mask (past the cache, unmapped pages) are
+        // zeroed: their probabilities are 0 but their bytes may not be finite.
+        const uint32_t rb = mask >> (16 * sb);
+        const uint32_t mlo = (((rb >> (2 * tg)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 1)) & 1u) ? 0xffff0000u : 0u);
+        const uint32_t mhi = (((rb >> (2 * tg + 8)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 9)) & 1u) ? 0xffff0000u : 0u);
+#pragma unroll
+        for (int mi = 0; mi < C::MT; ++mi) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_t(vt + swz_off<C::HALF_BYTES>(16 * sb + vrow, 16 * mi + vcol), a0, a1, a2, a3);
+          a0 &= mlo; a1 &= mlo; a2 &= mhi; a3 &= mhi;
+#pragma unroll
+          for (int nn = 0; nn < NT; ++nn) mma_bf16(acc[nn][mi], a0, a1, a2, a3, pb[sb][nn][0], pb[sb][nn][1]);
+        }
+      }
+      qf = qc + 2;
+      issue();
+    }
+    qc += text ? 2 : 1;
+  }
+  // After a timeout, let this warp's copies still in flight land (bounded)
+  // before the ring is reused below.
+  if (timed_out && lane == 0)
+    for (int q = max(qc, qi - S); q < qi; ++q) mbar_wait(full + q % S, (q / S) & 1);
+  __syncwarp();
+
+  // Warp statistics now; text outputs once every warp is done with the ring.
+#pragma unroll
+  for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+    for (int jj = 0; jj < 2; ++jj) {
+      const float a = group_sum(l1v[nn][jj]), bb = group_sum(ltv[nn][jj]);
+      const float cc = group_sum(l1t[nn][jj]), dd = group_sum(ltt[nn][jj]);
+      const int h = 8 * nn + 2 * tg + jj;
+      if (gr == 0) {
+        wst[warp][h][ST_MV] = m_v[nn][jj]; wst[warp][h][ST_L1V] = a; wst[warp][h][ST_LTV] = bb;
+        wst[warp][h][ST_MT] = m_t[nn][jj]; wst[warp][h][ST_L1T] = cc; wst[warp][h][ST_LTT] = dd;
+        wst[warp][h][3] = wst[warp][h][7] = 0.f;
+      }
+    }
+  pdl_trigger();
+  __syncthreads();
+  float* ow = reinterpret_cast<float*>(smem) + warp * GM * D;
+#pragma unroll
+  for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+    for (int mi = 0; mi < C::MT; ++mi) {
+      const int h0 = 8 * nn + 2 * tg, d0 = 16 * mi + gr;
+      ow[h0 * D + d0] = acc[nn][mi][0];
+      ow[(h0 + 1) * D + d0] = acc[nn][mi][1];
+      ow[h0 * D + d0 + 8] = acc[nn][mi][2];
+      ow[(h0 + 1) * D + d0 + 8] = acc[nn][mi][3];
+    }
+  if (timed_out) err |= ERR_TIMEOUT;
+  if (err) atomicOr(p.err, err);
+  score_epilogue<GM, D, NW, C::THREADS>(p, b, g, s, wst, reinterpret_cast<const float*>(smem), GM * D, tail);
 }
 
 // ---------------------------------------------------------------------------
@@ -1481,9 +1913,22 @@ size_t f32_smem() { return sizeof(F32Smem<D, GM>); }
 template <typename T, int D, int GM>
 size_t gather_smem() { return sizeof(GatherSmem<T, D, GM>); }
 
+// Warps per CTA and ring slots per warp of the bulk-tensor score kernel: two
+// CTAs (8 warps) share an SM, each warp with 24 KB of its tiles in flight.
+constexpr int kTmaWarps = 4;
+template <int D>
+constexpr int tma_slots() { return D == 128 ? 3 : 5; }
+template <int D, int NT>
+size_t tma_smem() { return TmaCfg<D, NT, kTmaWarps, tma_slots<D>()>::SMEM; }
+
 template <int D>
 cudaError_t launch_score_d(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.ns, p.Hkv, p.B);
+  if (p.dtype == 0 && p.use_tma) {
+    constexpr int NW = kTmaWarps, S = tma_slots<D>();
+    if (p.G <= 8) return launch_ex(k_score_tma<D, 1, NW, S>, grid, dim3(32 * NW), tma_smem<D, 1>(), st, 1, p);
+    return launch_ex(k_score_tma<D, 2, NW, S>, grid, dim3(32 * NW), tma_smem<D, 2>(), st, 1, p);
+  }
   if (p.dtype == 0) {
     if (p.G <= 8) return launch_ex(k_score_mma<D, 1>, grid, dim3(kThreads), mma_smem<D, 1>(), st, 1, p);
     return launch_ex(k_score_mma<D, 2>, grid, dim3(kThreads), mma_smem<D, 2>(), st, 1, p);
@@ -1518,6 +1963,10 @@ cudaError_t set_smem(void (*kernel)(StepParams), size_t bytes) {
 cudaError_t configure_fixed_kernels() {
   cudaError_t e = cudaSuccess;
 #define VP_SET(kernel, bytes) if (e == cudaSuccess) e = set_smem(kernel, bytes)
+  VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 1>()));
+  VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 2>()));
+  VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>()>), (tma_smem<64, 1>()));
+  VP_SET((k_score_tma<64, 2, kTmaWarps, tma_slots<64>()>), (tma_smem<64, 2>()));
   VP_SET((k_score_mma<128, 1>), (mma_smem<128, 1>()));
   VP_SET((k_score_mma<128, 2>), (mma_smem<128, 2>()));
   VP_SET((k_score_mma<64, 1>), (mma_smem<64, 1>()));
@@ -1575,6 +2024,85 @@ cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.cl, p.granularity ? p.Hkv : 1, p.B);
   return launch_ex(k_select, grid, dim3(kSelThreads), select_smem_bytes(p.max_visual, p.H, p.ns), st, p.cl, p);
+}
+
+namespace {
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      f = nullptr;
+    cudaGetLastError();
+    return reinterpret_cast<EncodeTiledFn>(f);
+  }();
+  return fn;
+}
+
+// 4-D descriptor of one cache: dims {D, token, kv-head, sequence or page}, the
+// last three ordered by increasing stride.  Returns false for a layout whose
+// extent along the token axis cannot be bounded by the caller's memory.
+bool encode_one(const KvView& kv, const StepParams& p, CUtensorMap* map, int* tpos, int* gpos, int* bpos) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || !kv.data) return false;
+  struct Ax { int64_t stride, size; int id; };  // id: 0 token, 1 kv-head, 2 sequence / page
+  Ax ax[3] = {{kv.st, 0, 0}, {kv.sh, p.Hkv, 1}, {kv.sb, p.paged ? kv.num_pages : p.B, 2}};
+  if (p.paged) ax[0].size = p.page_size;
+  for (int i = 0; i < 3; ++i)
+    for (int j = i + 1; j < 3; ++j)
+      if (ax[j].stride < ax[i].stride) { Ax t = ax[i]; ax[i] = ax[j]; ax[j] = t; }
+  if (ax[0].stride < p.D) return false;
+  if (!p.paged) {
+    // The token extent is the room its stride leaves before the next axis.
+    int k = 0;
+    while (ax[k].id != 0) ++k;
+    if (k == 2 || ax[k].stride <= 0) return false;
+    ax[k].size = ax[k + 1].stride / ax[k].stride;
+  }
+  for (int i = 0; i < 3; ++i) {
+    if (ax[i].size < 1 || ax[i].stride <= 0) return false;
+    if (i < 2 && ax[i + 1].stride < ax[i].stride * ax[i].size) return false;  // axes must nest
+  }
+  cuuint64_t dims[4] = {(cuuint64_t)p.D, (cuuint64_t)ax[0].size, (cuuint64_t)ax[1].size, (cuuint64_t)ax[2].size};
+  // Rows at or past max_seq are never read: the copy fills them with zeros.
+  for (int i = 0; i < 3; ++i)
+    if (!p.paged && ax[i].id == 0 && ax[i].size > p.max_seq) dims[i + 1] = (cuuint64_t)p.max_seq;
+  const cuuint64_t strides[3] = {(cuuint64_t)ax[0].stride * 2, (cuuint64_t)ax[1].stride * 2, (cuuint64_t)ax[2].stride * 2};
+  const int R = p.paged ? (p.page_size < kTmaTile ? p.page_size : kTmaTile) : kTmaTile;
+  cuuint32_t box[4] = {64, 1, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  for (int i = 0; i < 3; ++i) {
+    if (ax[i].id == 0) { box[i + 1] = (cuuint32_t)R; *tpos = i + 1; }
+    if (ax[i].id == 1) *gpos = i + 1;
+    if (ax[i].id == 2) *bpos = i + 1;
+  }
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(kv.data), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+}  // namespace
+
+void encode_kv_maps(StepParams& p) {
+  p.use_tma = 0;
+  if (p.dtype != 0 || (p.D != 64 && p.D != 128)) return;
+  if (p.paged) {
+    if (p.page_size < 8) return;  // box origins must stay 1024-byte aligned in shared memory
+    // Page ids of a CTA's boxes are staged in shared memory: bound them.
+    const int64_t tiles = (p.max_seq + kTmaTile - 1) / kTmaTile;
+    const int64_t per_cta = (2 * tiles + p.ns - 1) / p.ns + 1;
+    const int64_t boxes = per_cta * (kTmaTile / (p.page_size < kTmaTile ? p.page_size : kTmaTile));
+    if (boxes > kTmaMaxBoxes) return;
+  }
+  int kt = 0, kg = 0, kb = 0, vt = 0, vg = 0, vb = 0;
+  if (!encode_one(p.k, p, &p.tmk, &kt, &kg, &kb) || !encode_one(p.v, p, &p.tmv, &vt, &vg, &vb)) return;
+  if (kt != vt || kg != vg || kb != vb) return;  // both caches must share an axis order
+  p.tpos = kt; p.gpos = kg; p.bpos = kb;
+  p.use_tma = 1;
 }
 
 cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {

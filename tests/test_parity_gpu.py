@@ -97,6 +97,26 @@ def test_paged_cache_other_page_size(vp):
     Hn.check_all(vp, Hn.make_inputs(r), r.budget)
 
 
+@pytest.mark.parametrize("layout", Hn.LAYOUTS)
+@pytest.mark.parametrize("dtype,D", [(W.BF16, 128), (W.BF16, 64), (W.FP32, 128)])
+def test_cache_layouts(vp, layout, dtype, D):
+    """Dense, token-major, token-outermost and row-padded caches: the bulk
+    tensor copies serve the first, second and fourth, the per-row copies the
+    third; all must agree with the oracle."""
+    r = small(dtype=dtype, head_dim=D)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget, layout=layout)
+
+
+@pytest.mark.parametrize("page_size,layout", [(4, "bhtd"), (8, "bhtd"), (32, "bthd"), (64, "bhtd"),
+                                              (256, "bthd"), (16, "padded")])
+def test_paged_bf16_page_sizes(vp, page_size, layout):
+    """Pages smaller than, equal to and larger than the 32-token tile (below
+    8 tokens the per-row copies take over), in both pool layouts."""
+    r = small(batch=4, vis_len=(300, 577, 64, 1000), vis_start=(0, 13, 40, 0),
+              text_len=(517, 70, 129, 33), paged=True, page_size=page_size)
+    Hn.check_all(vp, Hn.make_inputs(r), r.budget, layout=layout)
+
+
 def test_explicit_logit_scale(vp):
     r = small()
     Hn.check_all(vp, Hn.make_inputs(r), dict(r.budget, scale=0.05))

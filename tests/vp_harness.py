@@ -53,10 +53,34 @@ def make_inputs(r: W.Recipe, layer=0, step=0, t_cap=None, q_override=None) -> In
     return inp
 
 
+LAYOUTS = ("bhtd", "bthd", "tbhd", "padded")
+
+
+def place(x: torch.Tensor, layout: str, dev) -> torch.Tensor:
+    """Device copy of a [B, Hkv, T, D] (or paged [P, Hkv, S, D]) cache viewed in
+    that logical order, with memory laid out as ``layout`` says:
+      bhtd    sequence, head, token, dim (dense);
+      bthd    sequence, token, head, dim (heads interleaved per token);
+      tbhd    token outermost (a layout the tensor-map path declines);
+      padded  bhtd with every row padded by 16 bytes."""
+    if layout == "bhtd":
+        return x.to(dev)
+    if layout == "bthd":
+        return x.permute(0, 2, 1, 3).contiguous().to(dev).permute(0, 2, 1, 3)
+    if layout == "tbhd":
+        return x.permute(2, 0, 1, 3).contiguous().to(dev).permute(1, 2, 0, 3)
+    if layout == "padded":
+        pad = 16 // x.element_size()
+        y = torch.full((*x.shape[:3], x.shape[3] + pad), float("nan"), dtype=x.dtype)
+        y[..., : x.shape[3]] = x
+        return y.to(dev)[..., : x.shape[3]]
+    raise ValueError(layout)
+
+
 class Device:
     """Device copies of an Inputs plus a library context and output buffers."""
 
-    def __init__(self, vp, inp: Inputs, budget: dict, max_batch=None, max_seq=None):
+    def __init__(self, vp, inp: Inputs, budget: dict, max_batch=None, max_seq=None, layout="bhtd"):
         self.vp = vp
         r = inp.recipe
         dev = torch.device("cuda")
@@ -72,11 +96,11 @@ class Device:
         if r.paged:
             pk = W.scatter_pages(inp.k, inp.block_table, inp.n_pages, r.page_size)
             pv = W.scatter_pages(inp.v, inp.block_table, inp.n_pages, r.page_size)
-            self.k_t, self.v_t = pk.to(dev), pv.to(dev)
+            self.k_t, self.v_t = place(pk, layout, dev), place(pv, layout, dev)
             self.bt = torch.from_numpy(inp.block_table).to(dev)
             self.kc, self.vc = vp.kv_paged(self.k_t, self.bt), vp.kv_paged(self.v_t, self.bt)
         else:
-            self.k_t, self.v_t = inp.k.to(dev), inp.v.to(dev)
+            self.k_t, self.v_t = place(inp.k, layout, dev), place(inp.v, layout, dev)
             self.kc, self.vc = vp.kv_contiguous(self.k_t), vp.kv_contiguous(self.v_t)
         self.vs = torch.from_numpy(inp.vis_start.astype(np.int32)).to(dev)
         self.vl = torch.from_numpy(inp.vis_len.astype(np.int32)).to(dev)
@@ -184,8 +208,8 @@ def compare_seq(inp: Inputs, gpu: dict, b: int, budget: dict, report: dict | Non
     return ref
 
 
-def check_all(vp, inp: Inputs, budget: dict, seqs=None, report=None):
-    dev = Device(vp, inp, budget)
+def check_all(vp, inp: Inputs, budget: dict, seqs=None, report=None, layout="bhtd"):
+    dev = Device(vp, inp, budget, layout=layout)
     try:
         gpu = dev.run()
     finally:
