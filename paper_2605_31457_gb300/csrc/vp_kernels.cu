@@ -20,9 +20,13 @@
 // Logits are carried in log2 units (z * log2 e) so that every exponential is
 // one exp2f: exp(z - m) = exp2(z2 - m2), exp((z - m) / tau) = exp2((z2 - m2) / tau).
 //
-// Every kernel starts with griddepcontrol.wait, so it may be launched as a
-// programmatic dependent of the preceding kernel on the stream: it reads no
-// input before that kernel has completed and its writes are visible.
+// Every kernel may be launched as a programmatic dependent of the preceding
+// kernel on the stream: it reads nothing that kernel writes before
+// griddepcontrol.wait.  The slice gather kernel reads the call's inputs and
+// the score kernel's partials before its wait: the select kernel between them
+// lets its dependents start only after its own wait on the score kernel, so
+// both are complete by then.  Each kernel also lets its own dependent start
+// only after that wait, so the next call cannot overwrite the workspace early.
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -40,7 +44,7 @@ constexpr int kWarps = 8;                 // warps of a score CTA
 constexpr int kThreads = 32 * kWarps;
 constexpr int kStages = 3;                // TMA ring depth per warp
 constexpr int kTile = 16;                 // tokens per tile
-constexpr int kSelThreads = 1024;
+constexpr int kSelSliceSmall = 2048;  // longest slice per select rank for 512 threads
 constexpr int kMaxHeads = 128;
 constexpr int kGatherThreads = 256;
 constexpr int kGatherWarps = kGatherThreads / 32;
@@ -1178,9 +1182,9 @@ __global__ void __launch_bounds__(kThreads) k_score_f32(const __grid_constant__ 
 }
 
 // ---------------------------------------------------------------------------
-// k_select: grid (cl, granularity ? Hkv : 1, B) in clusters of cl CTAs,
-// 1024 threads.  Dynamic shared memory: rank 0 holds the N_v score keys; every
-// rank stages the split statistics after them.
+// k_select: grid (cl, granularity ? Hkv : 1, B) in clusters of cl CTAs of
+// 512 threads (1024 when a rank's slice of the visual tokens is long).
+// Dynamic shared memory: the N_v score keys, of which rank 0's copy is used.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int budget_k(const StepParams& p, float m_max, int nv) {
   if (nv <= 0) return 0;
@@ -1229,8 +1233,10 @@ __device__ __forceinline__ int block_excl_scan(int x, int* wsum_s) {
   return res;
 }
 
-__global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ StepParams p) {
-  extern __shared__ __align__(16) uint32_t key_s[];  // [max_visual] keys, then [H][ns][ST_N] statistics
+template <int NTH>
+__global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepParams p) {
+  constexpr int NW = NTH / 32;
+  extern __shared__ __align__(16) uint32_t key_s[];  // [max_visual] score keys (rank 0's copy is used)
   __shared__ float hM_s[kMaxHeads], hInv_s[kMaxHeads], hMass_s[kMaxHeads], hMass1_s[kMaxHeads];
   __shared__ unsigned hist_s[256];
   __shared__ int wsum_s[32];
@@ -1238,51 +1244,76 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
+  const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < 256; i += NTH) hist_s[i] = 0;
   pdl_wait();
   pdl_trigger();
-  const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31;
   const int H = p.H, ns = p.ns;
+  const float inv_tau = p.inv_tau;
+
+  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5, Eq. 6).
+  //    Warp w merges heads w, w + NW, ...; lane l folds splits l, l + 32, ...
+  //    in a running (max, sums) state and the warp merges the lanes.  The
+  //    first records are requested together with the sequence lengths, and
+  //    each head's records while the previous head is being merged.
+  const float* stb = p.split_st + (int64_t)b * H * p.nsp_max * ST_N;
+  auto fetch = [&](int h, int s, float4& x, float4& y) {  // x: text (M, L1, Ltau), y: visual
+    if (h < H && s < ns) {
+      const float4* r = reinterpret_cast<const float4*>(stb + ((int64_t)h * p.nsp_max + s) * ST_N);
+      x = __ldcg(r);
+      y = __ldcg(r + 1);
+    } else {
+      x = y = make_float4(-CUDART_INF_F, 0.f, 0.f, 0.f);
+    }
+  };
+  float4 cx0, cy0, cx1, cy1;
+  fetch(warp, lane, cx0, cy0);
+  fetch(warp, lane + 32, cx1, cy1);
   const Seq sq = load_seq(p, b, false);
   const int nv = sq.nv;
-  float* st_s = reinterpret_cast<float*>(key_s + ((p.max_visual + 3) & ~3));
-
-  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5, Eq. 6):
-  //    staged with one parallel load, then merged per head.
-  for (int i = tid; i < H * ns * 2; i += kSelThreads) {
-    const int h = i / (2 * ns), sp = (i >> 1) % ns, half = i & 1;
-    *reinterpret_cast<float4*>(st_s + (h * ns + sp) * ST_N + 4 * half) = __ldcg(
-        reinterpret_cast<const float4*>(p.split_st + (((int64_t)b * H + h) * p.nsp_max + sp) * ST_N + 4 * half));
-  }
-  // The first logit row of this thread's slice is fetched now, while the
-  // statistics are still in flight (heads up to 32).
+  // This rank's slice of the visual tokens; its first logit row is requested
+  // now so that it arrives while the statistics are merged (heads up to 32;
+  // at 1024 threads the registers are too few for it).
   const int per = (nv + ncl - 1) / ncl;
   const int i0 = min(nv, rank * per), i1 = min(nv, i0 + per);
   const int hbeg = p.granularity ? gsel * p.G : 0;
   const int hcnt = p.granularity ? p.G : H;
   const bool vec = (hbeg & 3) == 0 && (hcnt & 3) == 0;
-  const bool pre = vec && hcnt <= 32 && i0 + tid < i1;
+  const bool pre = NTH <= 512 && vec && hcnt <= 32 && i0 + tid < i1;
   float4 zpre[8];
   if (pre) {
     const float4* zr = reinterpret_cast<const float4*>(p.z_ws + ((int64_t)b * p.max_visual + i0 + tid) * p.hp + hbeg);
 #pragma unroll
     for (int q = 0; q < 8; ++q) zpre[q] = 4 * q < hcnt ? __ldcg(zr + q) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  __syncthreads();
-  // One warp per head, lanes over the splits.
-  for (int h = tid >> 5; h < H; h += kSelThreads / 32) {
-    const float* st = st_s + h * ns * ST_N;
-    float M = -CUDART_INF_F;
-    for (int s = lane; s < ns; s += 32) M = fmaxf(M, fmaxf(st[s * ST_N + ST_MV], st[s * ST_N + ST_MT]));
-    M = warp_max(M);
-    float L1v = 0.f, L1t = 0.f, Ltv = 0.f, Ltt = 0.f;
-    for (int s = lane; s < ns; s += 32) {
-      const float* r = st + s * ST_N;
-      L1v += exp2_rel(r[ST_MV], M) * r[ST_L1V];
-      Ltv += exp2_tau(r[ST_MV], M, p.inv_tau) * r[ST_LTV];
-      L1t += exp2_rel(r[ST_MT], M) * r[ST_L1T];
-      Ltt += exp2_tau(r[ST_MT], M, p.inv_tau) * r[ST_LTT];
+  for (int h = warp; h < H; h += NW) {
+    float4 nx0, ny0, nx1, ny1;
+    fetch(h + NW, lane, nx0, ny0);
+    fetch(h + NW, lane + 32, nx1, ny1);
+    float m = -CUDART_INF_F, a1v = 0.f, atv = 0.f, a1t = 0.f, att = 0.f;
+    auto fold = [&](const float4& x, const float4& y) {
+      const float mn = fmaxf(m, fmaxf(x.x, y.x));
+      if (mn > m) {
+        const float f1 = exp2_rel(m, mn), ft = exp2_tau(m, mn, inv_tau);
+        a1v *= f1; a1t *= f1; atv *= ft; att *= ft;
+        m = mn;
+      }
+      a1v = fmaf(exp2_rel(y.x, m), y.y, a1v);
+      atv = fmaf(exp2_tau(y.x, m, inv_tau), y.z, atv);
+      a1t = fmaf(exp2_rel(x.x, m), x.y, a1t);
+      att = fmaf(exp2_tau(x.x, m, inv_tau), x.z, att);
+    };
+    fold(cx0, cy0);
+    fold(cx1, cy1);
+    for (int s = lane + 64; s < ns; s += 32) {
+      float4 x, y;
+      fetch(h, s, x, y);
+      fold(x, y);
     }
-    L1v = warp_sum(L1v); Ltv = warp_sum(Ltv); L1t = warp_sum(L1t); Ltt = warp_sum(Ltt);
+    const float M = warp_max(m);
+    const float f1 = exp2_rel(m, M), ft = exp2_tau(m, M, inv_tau);
+    const float L1v = warp_sum(a1v * f1), Ltv = warp_sum(atv * ft);
+    const float L1t = warp_sum(a1t * f1), Ltt = warp_sum(att * ft);
     if (lane == 0) {
       const float L1 = L1v + L1t, Lt = Ltv + Ltt;
       hM_s[h] = M;
@@ -1290,15 +1321,43 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
       hMass_s[h] = Lt > 0.f ? Ltv / Lt : 0.f;
       hMass1_s[h] = L1 > 0.f ? L1v / L1 : 0.f;
     }
+    cx0 = nx0; cy0 = ny0; cx1 = nx1; cy1 = ny1;
   }
   __syncthreads();
 
-  // 2. Importance S_i (Eq. 2) of this rank's slice of the visual tokens, as
+  // 2. Rank 0: head mean, head max (Sec. 4.3) and the budget (Eq. 7).
+  const int nsel = p.granularity ? p.Hkv : 1;
+  if (rank == 0) {
+    if (warp == 0) {
+      float sm = 0.f, mx = 0.f, s1 = 0.f;
+      for (int h = lane; h < H; h += 32) {
+        sm += hMass_s[h];
+        mx = fmaxf(mx, hMass_s[h]);
+        s1 += hMass1_s[h];
+      }
+      sm = warp_sum(sm);
+      mx = warp_max(mx);
+      s1 = warp_sum(s1);
+      if (lane == 0) {
+        const int K = min(budget_k(p, mx, nv), p.kept_cap);
+        sh_i[0] = K;
+        p.kept_count[(int64_t)b * nsel + gsel] = K;
+        if (gsel == 0 && p.mass_stats) {
+          float* ms = p.mass_stats + (int64_t)b * 4;
+          ms[0] = sm / H; ms[1] = mx; ms[2] = s1 / H; ms[3] = (float)K;
+        }
+      }
+    } else if (gsel == 0) {
+      for (int h = tid - 32; h < H; h += NTH - 32) p.mass[(int64_t)b * H + h] = hMass_s[h];
+    }
+  }
+
+  // 3. Importance S_i (Eq. 2) of this rank's slice of the visual tokens, as
   //    float bits (S >= 0 orders like its bits), into rank 0's key array.
   const float inv_cnt = 1.f / (float)hcnt;
   uint32_t* key0 = ncl > 1 ? cluster.map_shared_rank(key_s, 0) : key_s;
   unsigned bad = 0;
-  for (int i = i0 + tid; i < i1; i += kSelThreads) {
+  for (int i = i0 + tid; i < i1; i += NTH) {
     const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
     float a = 0.f;
     if (pre && i == i0 + tid) {
@@ -1330,42 +1389,16 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     key0[i] = __float_as_uint(sc);
   }
   if (bad) atomicOr(p.err, ERR_NONFINITE);
-  if (ncl > 1) cluster.sync();  // rank 0 now sees every key
+  if (ncl > 1) cluster.sync();  // rank 0 now sees every key (and its own K)
   else __syncthreads();
   if (rank != 0) return;
 
-  // 3. Head mean, head max (Sec. 4.3) and the budget (Eq. 7).
-  if (tid < 32) {
-    float sm = 0.f, mx = 0.f, s1 = 0.f;
-    for (int h = tid; h < H; h += 32) {
-      sm += hMass_s[h];
-      mx = fmaxf(mx, hMass_s[h]);
-      s1 += hMass1_s[h];
-    }
-    sm = warp_sum(sm);
-    mx = warp_max(mx);
-    s1 = warp_sum(s1);
-    if (tid == 0) {
-      const int K = min(budget_k(p, mx, nv), p.kept_cap);
-      sh_i[0] = K;
-      sh_i[1] = 0;
-      sh_i[2] = 0;
-      if (gsel == 0 && p.mass_stats) {
-        float* ms = p.mass_stats + (int64_t)b * 4;
-        ms[0] = sm / H; ms[1] = mx; ms[2] = s1 / H; ms[3] = (float)K;
-      }
-    }
-  }
-  if (gsel == 0)
-    for (int h = tid; h < H; h += kSelThreads) p.mass[(int64_t)b * H + h] = hMass_s[h];
-  __syncthreads();
   const int K = sh_i[0];
-  const int nsel = p.granularity ? p.Hkv : 1;
   int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
-  if (tid == 0) p.kept_count[(int64_t)b * nsel + gsel] = K;
 
   // 4. Radix select of the K-th largest key, 8 bits per pass from the top;
-  //    lanes holding the same digit add to the histogram once per warp.
+  //    lanes holding the same digit add to the histogram once per warp.  Warp
+  //    0 scans the histogram and clears it for the next pass.
   const bool take_all = K >= nv;
   uint32_t theta = 0;
   unsigned krem = 0, n_theta = 0;  // keys equal to theta: to keep, in total
@@ -1373,15 +1406,11 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
     uint32_t prefix = 0, mask = 0;
     krem = (unsigned)K;
     for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int i = tid; i < 256; i += kSelThreads) hist_s[i] = 0;
-      __syncthreads();
-      for (int base = 0; base < nv; base += kSelThreads) {
+      for (int base = 0; base < nv; base += NTH) {
         const int i = base + tid;
         const uint32_t k = i < nv ? key_s[i] : 0u;
         const bool m = i < nv && (k & mask) == prefix;
         const unsigned dg = (k >> shift) & 255u;
-        // One atomic per warp when all its candidates share the digit (the
-        // common case in the upper passes); one per lane otherwise.
         const unsigned act = __ballot_sync(0xffffffffu, m);
         if (act) {
           const int leader = __ffs(act) - 1;
@@ -1394,23 +1423,32 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
         }
       }
       __syncthreads();
-      if (tid < 32) {
+      if (warp == 0) {
         // Lane L owns digits 255-8L ... 248-8L (descending).
         unsigned c[8], tot = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) { c[j] = hist_s[255 - 8 * tid - j]; tot += c[j]; }
+        for (int j = 0; j < 8; ++j) {
+          c[j] = hist_s[255 - 8 * lane - j];
+          hist_s[255 - 8 * lane - j] = 0;
+          tot += c[j];
+        }
         unsigned incl = tot;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
           const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
-          if (tid >= o) incl += n;
+          if (lane >= o) incl += n;
         }
         const unsigned excl = incl - tot;
         if (excl < krem && krem <= incl) {
           unsigned run = excl;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            if (run + c[j] >= krem) { sh_i[1] = 255 - 8 * tid - j; sh_i[2] = (int)run; break; }
+            if (run + c[j] >= krem) {
+              sh_i[1] = 255 - 8 * lane - j;
+              sh_i[2] = (int)run;
+              sh_i[3] = (int)c[j];
+              break;
+            }
             run += c[j];
           }
         }
@@ -1419,8 +1457,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
       krem -= (unsigned)sh_i[2];
       prefix |= (uint32_t)sh_i[1] << shift;
       mask |= 255u << shift;
-      if (shift == 0) n_theta = hist_s[sh_i[1]];
-      __syncthreads();
+      if (shift == 0) n_theta = (unsigned)sh_i[3];
     }
     theta = prefix;  // the K-th largest key; krem keys equal to it are kept
   }
@@ -1428,7 +1465,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
   // 5. Ascending compaction: keys above theta, plus the first krem equal keys
   //    (every equal key when there is no tie to break: one scan less).
   if (K > 0) {
-    const int per_t = (nv + kSelThreads - 1) / kSelThreads;
+    const int per_t = (nv + NTH - 1) / NTH;
     const int j0 = min(nv, tid * per_t), j1 = min(nv, j0 + per_t);
     const bool ties = !take_all && krem < n_theta;
     int n_eq = 0;
@@ -1455,7 +1492,7 @@ __global__ void __launch_bounds__(kSelThreads) k_select(const __grid_constant__ 
       if (sel && o < K) kept[o++] = i;
     }
   }
-  for (int i = max(K, 0) + tid; i < p.kept_cap; i += kSelThreads) kept[i] = -1;
+  for (int i = max(K, 0) + tid; i < p.kept_cap; i += NTH) kept[i] = -1;
 }
 
 // ---------------------------------------------------------------------------
@@ -1714,22 +1751,24 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // ---------------------------------------------------------------------------
 // k_gather_slice: grid (D / 16, Hkv, B), 256 threads, for kept sets of at most
 // kSliceMaxKept tokens per (sequence, kv-head).  CTA c owns output dimensions
-// [16c, 16c + 16) of the G heads: warps 0-3 attend over every kept visual
-// token (reading only their 16-dimension slice of V), warps 4-7 merge the same
-// slice of the score splits' text partials, and the CTA combines both in
-// log-sum-exp form.  No partial leaves the CTA.
+// [16c, 16c + 16) of the G heads.  It first merges the same slice of the
+// score splits' text partials -- they come from the score kernel, which has
+// completed before any select CTA lets this grid start, so this part runs
+// before griddepcontrol.wait and overlaps the select kernel.  After the wait
+// it attends over every kept visual token (reading only its 16-dimension
+// slice of V, fetched in the same round trip as the token's logits) and
+// combines both parts in log-sum-exp form.  No partial leaves the CTA.
 // ---------------------------------------------------------------------------
 constexpr int kSliceMaxKept = 256;
 constexpr int kSliceDims = 16;
 
 template <int GM>
 struct SliceSmem {
-  int idx[kSliceMaxKept];
   float pz[GM][kSliceMaxKept];            // kept logits, then probabilities
   float tm[GM][kNsMax];                   // text split maxima, then weights
   float tl[GM][kNsMax];                   // text split sums
-  float red[4][GM][kSliceDims];           // kept-part warp partials
-  float4 tred[128];                       // text-part thread partials
+  float red[kGatherWarps][GM][kSliceDims];  // kept-part warp partials
+  float4 tred[kGatherThreads];            // text-part thread partials
   float fin[GM][4];                       // m_k, l_k, M_t, L_t
 };
 
@@ -1738,34 +1777,17 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
   constexpr int SD = kSliceDims;
   constexpr int CH = 16 / sizeof(T);      // elements per 16-byte chunk
   constexpr int CPS = SD / CH;            // chunks per row slice (2 bf16, 4 fp32)
-  constexpr int TSTRIDE = 128 / CPS;      // kept tokens handled side by side
+  constexpr int TSTRIDE = kGatherThreads / CPS;  // kept tokens handled side by side
+  constexpr int TPT = kSliceMaxKept / TSTRIDE;   // kept tokens per thread
   extern __shared__ __align__(16) unsigned char smem_raw[];
   auto& sm = *reinterpret_cast<SliceSmem<GM>*>(smem_raw);
   const int cd = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-  pdl_wait();
-  pdl_trigger();
   const int G = p.G, H = p.H, ns = p.ns;
   const int64_t hrow0 = (int64_t)b * H + g * G;
   const Seq sq = load_seq(p, b, false);
-  const int sel = p.granularity ? b * p.Hkv + g : b;
-  const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, min(p.kept_cap, kSliceMaxKept))));
-  const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
-  unsigned err = 0;
 
-  // 1. Kept indices and their logits; text split statistics (one round trip).
-  for (int t = tid; t < K; t += kGatherThreads) {
-    int i = __ldg(kept + t);
-    if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
-    sm.idx[t] = i;
-    const float* zr = p.z_ws + ((int64_t)b * p.max_visual + (i < 0 ? 0 : i)) * p.hp + g * G;
-    float zv[GM];
-#pragma unroll
-    for (int h = 0; h < GM; ++h) zv[h] = (i >= 0 && h < G) ? __ldcg(zr + h) : -CUDART_INF_F;
-#pragma unroll
-    for (int h = 0; h < GM; ++h) sm.pz[h][t] = zv[h];
-  }
+  // 1. Text split statistics, then per head: text max, split weights, sum.
   for (int i = tid; i < G * ns; i += kGatherThreads) {
     const int h = i / ns, s = i % ns;
     const float2 r = __ldcg(reinterpret_cast<const float2*>(p.split_st + ((hrow0 + h) * p.nsp_max + s) * ST_N));
@@ -1773,8 +1795,82 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
     sm.tl[h][s] = r.y;  // ST_L1T
   }
   __syncthreads();
+  for (int h = warp; h < G; h += kGatherWarps) {
+    float mt = -CUDART_INF_F;
+    for (int s = lane; s < ns; s += 32) mt = fmaxf(mt, sm.tm[h][s]);
+    mt = warp_max(mt);
+    float lt = 0.f;
+    for (int s = lane; s < ns; s += 32) {
+      const float w = exp2_rel(sm.tm[h][s], mt);
+      sm.tm[h][s] = w;
+      lt = fmaf(w, sm.tl[h][s], lt);
+    }
+    lt = warp_sum(lt);
+    if (lane == 0) { sm.fin[h][2] = mt; sm.fin[h][3] = lt; }
+  }
+  __syncthreads();
+  // 2. Text partials of the slice: thread (element e = (head, float4), split group sg).
+  {
+    const int NE = G * (SD / 4);
+    const int nsg = kGatherThreads / NE;
+    const int e = tid % NE, sg = tid / NE;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (sg < nsg) {
+      const int h = e / (SD / 4), d = cd * SD + 4 * (e % (SD / 4));
+      const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
+#pragma unroll 4
+      for (int s = sg; s < ns; s += nsg) {
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
+        const float w = sm.tm[h][s];
+        acc.x = fmaf(w, v.x, acc.x); acc.y = fmaf(w, v.y, acc.y); acc.z = fmaf(w, v.z, acc.z); acc.w = fmaf(w, v.w, acc.w);
+      }
+    }
+    sm.tred[tid] = acc;
+  }
 
-  // 2. Per head: kept max / probabilities / sum, text max / weights / sum.
+  pdl_wait();
+  pdl_trigger();
+  const int sel = p.granularity ? b * p.Hkv + g : b;
+  const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, min(p.kept_cap, kSliceMaxKept))));
+  const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
+  unsigned err = 0;
+
+  // 3. Kept tokens: thread (token slot j0, chunk q) takes tokens j0 + TSTRIDE t;
+  //    their V slices and (chunk 0) their logits are fetched together.
+  const int j0 = tid / CPS, q = tid % CPS;
+  int idx[TPT];
+#pragma unroll
+  for (int t = 0; t < TPT; ++t) {
+    const int j = j0 + TSTRIDE * t;
+    idx[t] = j < K ? __ldg(kept + j) : -1;
+    if (j < K && (idx[t] < 0 || idx[t] >= sq.nv)) { err |= ERR_KEPT; idx[t] = -1; }
+  }
+  float vv[TPT][CH];
+#pragma unroll
+  for (int t = 0; t < TPT; ++t) {
+#pragma unroll
+    for (int e = 0; e < CH; ++e) vv[t][e] = 0.f;
+    if (idx[t] >= 0) {
+      const T* vr = kv_row<T>(p.v, p, b, g, sq.vs + idx[t]);
+      if (vr) load_f<CH>(vr + cd * SD + q * CH, vv[t]);
+      else err |= ERR_PAGE;
+    }
+  }
+  if (q == 0) {
+#pragma unroll
+    for (int t = 0; t < TPT; ++t) {
+      const int j = j0 + TSTRIDE * t;
+      if (j >= K) break;
+      const float* zr = p.z_ws + ((int64_t)b * p.max_visual + (idx[t] < 0 ? 0 : idx[t])) * p.hp + g * G;
+      float zv[GM];
+#pragma unroll
+      for (int h = 0; h < GM; ++h) zv[h] = (idx[t] >= 0 && h < G) ? __ldcg(zr + h) : -CUDART_INF_F;
+#pragma unroll
+      for (int h = 0; h < GM; ++h) sm.pz[h][j] = zv[h];
+    }
+  }
+  __syncthreads();
+  // 4. Per head: kept max, probabilities, sum.
   for (int h = warp; h < G; h += kGatherWarps) {
     float m = -CUDART_INF_F;
     for (int t = lane; t < K; t += 32) m = fmaxf(m, sm.pz[h][t]);
@@ -1786,42 +1882,26 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
       l += e;
     }
     l = warp_sum(l);
-    float mt = -CUDART_INF_F;
-    for (int s = lane; s < ns; s += 32) mt = fmaxf(mt, sm.tm[h][s]);
-    mt = warp_max(mt);
-    float lt = 0.f;
-    for (int s = lane; s < ns; s += 32) {
-      const float w = exp2_rel(sm.tm[h][s], mt);
-      sm.tm[h][s] = w;
-      lt = fmaf(w, sm.tl[h][s], lt);
-    }
-    lt = warp_sum(lt);
-    if (lane == 0) { sm.fin[h][0] = m; sm.fin[h][1] = l; sm.fin[h][2] = mt; sm.fin[h][3] = lt; }
+    if (lane == 0) { sm.fin[h][0] = m; sm.fin[h][1] = l; }
   }
   __syncthreads();
-
-  float ko[GM][CH];  // kept part (warps 0-3)
-  if (warp < 4) {
-    // 3a. Kept tokens: thread (token j, chunk q) of the slice.
-    const int j0 = tid / CPS, q = tid % CPS;
+  // 5. P.V over the kept tokens from registers, reduced over the warp's token lanes.
+  {
+    float ko[GM][CH];
 #pragma unroll
     for (int h = 0; h < GM; ++h)
 #pragma unroll
       for (int e = 0; e < CH; ++e) ko[h][e] = 0.f;
-#pragma unroll 4
-    for (int j = j0; j < K; j += TSTRIDE) {
-      const int i = sm.idx[j];
-      if (i < 0) continue;
-      const T* vr = kv_row<T>(p.v, p, b, g, sq.vs + i);
-      if (!vr) { err |= ERR_PAGE; continue; }
-      float vv[CH];
-      load_f<CH>(vr + cd * SD + q * CH, vv);
+#pragma unroll
+    for (int t = 0; t < TPT; ++t) {
+      const int j = j0 + TSTRIDE * t;
+      if (j >= K) break;
 #pragma unroll
       for (int h = 0; h < GM; ++h) {
         if (h >= G) break;
         const float pr = sm.pz[h][j];
 #pragma unroll
-        for (int e = 0; e < CH; ++e) ko[h][e] = fmaf(pr, vv[e], ko[h][e]);
+        for (int e = 0; e < CH; ++e) ko[h][e] = fmaf(pr, vv[t][e], ko[h][e]);
       }
     }
 #pragma unroll
@@ -1836,35 +1916,17 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
 #pragma unroll
         for (int e = 0; e < CH; ++e) sm.red[warp][h][lane * CH + e] = ko[h][e];
     }
-  } else {
-    // 3b. Text partials: thread (element e = (head, float4), split group sg).
-    const int u = tid - 128;
-    const int NE = G * (SD / 4);
-    const int nsg = 128 / NE;
-    const int e = u % NE, sg = u / NE;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (sg < nsg) {
-      const int h = e / (SD / 4), d = cd * SD + 4 * (e % (SD / 4));
-      const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
-#pragma unroll 4
-      for (int s = sg; s < ns; s += nsg) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
-        const float w = sm.tm[h][s];
-        acc.x = fmaf(w, v.x, acc.x); acc.y = fmaf(w, v.y, acc.y); acc.z = fmaf(w, v.z, acc.z); acc.w = fmaf(w, v.w, acc.w);
-      }
-    }
-    sm.tred[u] = acc;
   }
   if (err) atomicOr(p.err, err);
   __syncthreads();
 
-  // 4. Combine (thread per (head, dimension) of the slice).
+  // 6. Combine (thread per (head, dimension) of the slice).
   if (tid < G * SD) {
     const int h = tid / SD, d = tid % SD;
     float kv = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) kv += sm.red[w][h][d];
-    const int NE = G * (SD / 4), nsg = 128 / NE;
+    for (int w = 0; w < kGatherWarps; ++w) kv += sm.red[w][h][d];
+    const int NE = G * (SD / 4), nsg = kGatherThreads / NE;
     const int e = h * (SD / 4) + d / 4;
     float tv = 0.f;
     for (int sg = 0; sg < nsg; ++sg) {
@@ -2005,9 +2067,7 @@ cudaError_t configure_fixed_kernels() {
   return e;
 }
 
-size_t select_smem_bytes(int max_visual, int H, int ns) {
-  return ((size_t)(max_visual > 0 ? max_visual : 1) + 3) / 4 * 16 + (size_t)H * ns * ST_N * sizeof(float);
-}
+size_t select_smem_bytes(int max_visual) { return ((size_t)(max_visual > 0 ? max_visual : 1) + 3) / 4 * 16; }
 
 }  // namespace
 
@@ -2023,7 +2083,9 @@ cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
 
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.cl, p.granularity ? p.Hkv : 1, p.B);
-  return launch_ex(k_select, grid, dim3(kSelThreads), select_smem_bytes(p.max_visual, p.H, p.ns), st, p.cl, p);
+  const size_t smem = select_smem_bytes(p.max_visual);
+  if ((p.max_visual + p.cl - 1) / p.cl <= kSelSliceSmall) return launch_ex(k_select<512>, grid, dim3(512), smem, st, p.cl, p);
+  return launch_ex(k_select<1024>, grid, dim3(1024), smem, st, p.cl, p);
 }
 
 namespace {
@@ -2106,11 +2168,15 @@ void encode_kv_maps(StepParams& p) {
 }
 
 cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {
-  cudaFuncAttributes attr;
-  cudaError_t e = cudaFuncGetAttributes(&attr, k_select);
-  if (e != cudaSuccess) return e;
-  const int need = (int)select_smem_bytes(max_visual, H, nsp_max);
-  if (attr.maxDynamicSharedSizeBytes < need) e = set_smem(k_select, need);
+  (void)H;
+  (void)nsp_max;
+  const int need = (int)select_smem_bytes(max_visual);
+  cudaError_t e = cudaSuccess;
+  for (void (*k)(StepParams) : {k_select<512>, k_select<1024>}) {
+    cudaFuncAttributes attr;
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k);
+    if (e == cudaSuccess && attr.maxDynamicSharedSizeBytes < need) e = set_smem(k, need);
+  }
   return e == cudaSuccess ? configure_fixed_kernels() : e;
 }
 
