@@ -27,6 +27,7 @@ struct vp_ctx {
   float* gpart_st = nullptr;
   float* mt_o = nullptr;
   float* mt_st = nullptr;
+  float* hmax = nullptr;
   unsigned* tickets = nullptr;
   unsigned* err = nullptr;
   std::string last_error;
@@ -178,6 +179,7 @@ vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx) {
   ctx->gpart_st = reinterpret_cast<float*>(base + L.o_gs);
   ctx->mt_o = reinterpret_cast<float*>(base + L.o_mo);
   ctx->mt_st = reinterpret_cast<float*>(base + L.o_ms);
+  ctx->hmax = reinterpret_cast<float*>(base + L.o_hm);
   ctx->tickets = reinterpret_cast<unsigned*>(base + L.o_tickets);
   ctx->err = reinterpret_cast<unsigned*>(base + L.o_err);
   e = cudaMemset(ctx->ws, 0, ctx->ws_bytes);
@@ -254,7 +256,7 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   p.ns = pl.ns; p.nsp_max = ctx->lay.nsp_max; p.cl = pl.cl;
   p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
   vp::encode_kv_maps(p);
-  p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st;
+  p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st; p.hmax = ctx->hmax;
 
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   cudaEvent_t* tev = nullptr;

@@ -68,6 +68,7 @@ struct StepParams {
   float* gpart_st;    // [max_batch][Hkv][nk_max][G][2] {max, sum}
   float* mt_o;        // [max_batch][H][D] text output merged over the splits
   float* mt_st;       // [max_batch][H][2] its {max, sum}
+  float* hmax;        // [max_batch][H] largest logit of every head over all tokens (log2 units)
   unsigned* tickets;  // [max_batch][Hkv] (zero between calls)
   unsigned* err;      // device error word
   int hp;             // z_ws row stride (H rounded up to a multiple of 4)
@@ -87,7 +88,7 @@ constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
 
 // Launch plan of one call: score CTAs sized to the work (see below),
 // select clusters that spread the importance scores of few sequences over
-// several SMs, gather chunks of about 256 kept rows.
+// several SMs, gather chunks of 256 to 1024 kept rows.
 struct Plan {
   int ns, cl, nk, nm, nc, gslice;
 };
@@ -115,7 +116,11 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   const long long sel = (long long)batch * (granularity ? Hkv : 1);
   int cl = 1;
   while (cl < 8 && sel * cl * 2 <= num_sms) cl *= 2;
-  long long nk = (kept_cap + 255) / 256;
+  // Kept chunks of about 1024 rows, smaller (down to 256) while the gather
+  // grid would not fill the GPU twice.
+  long long nk = (kept_cap + 1023) / 1024;
+  const long long nk_want = (2 * slots + units - 1) / units, nk_small = (kept_cap + 255) / 256;
+  if (nk < nk_want) nk = nk_want < nk_small ? nk_want : nk_small;
   if (nk < 1) nk = 1;
   if (nk > kNkMax) nk = kNkMax;
   const int nm = ns > 1 ? (D / 16 < kMaxMerge ? D / 16 : kMaxMerge) : 0;
@@ -125,7 +130,7 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
 // Workspace layout for up to `batch` sequences (offsets in bytes, 256-aligned).
 // The first `zero_bytes` (tickets, error word) must be zero before a call.
 struct WsLayout {
-  size_t o_tickets, o_err, zero_bytes, o_z, o_st, o_o, o_go, o_gs, o_mo, o_ms, total;
+  size_t o_tickets, o_err, zero_bytes, o_z, o_st, o_o, o_go, o_gs, o_mo, o_ms, o_hm, total;
   int hp, nsp_max, nk_max;
 };
 
@@ -152,6 +157,7 @@ inline WsLayout ws_layout(int batch, int H, int Hkv, int D, int max_visual, int 
   w.o_gs = off; off = ws_round(off + B * Hkv * (size_t)w.nk_max * G * 2 * 4);
   w.o_mo = off; off = ws_round(off + B * H * (size_t)D * 4);
   w.o_ms = off; off = ws_round(off + B * H * 2 * 4);
+  w.o_hm = off; off = ws_round(off + B * H * 4);
   w.total = off;
   return w;
 }

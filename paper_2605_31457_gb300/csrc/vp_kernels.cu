@@ -199,6 +199,19 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, unsigned by
                ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
 }
 
+// 16- and 4-byte asynchronous copies global -> shared (LSU path), and the
+// arrive-on that completes an mbarrier phase once this thread's earlier such
+// copies have landed (the barrier's count must include these arrivals).
+__device__ __forceinline__ void cp_async16(unsigned dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(unsigned dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_arrive(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
+
 struct Seq {
   int vs, nv, tl;
 };
@@ -1348,7 +1361,10 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
         }
       }
     } else if (gsel == 0) {
-      for (int h = tid - 32; h < H; h += NTH - 32) p.mass[(int64_t)b * H + h] = hMass_s[h];
+      for (int h = tid - 32; h < H; h += NTH - 32) {
+        p.mass[(int64_t)b * H + h] = hMass_s[h];
+        p.hmax[(int64_t)b * H + h] = hM_s[h];
+      }
     }
   }
 
@@ -1495,6 +1511,108 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   for (int i = max(K, 0) + tid; i < p.kept_cap; i += NTH) kept[i] = -1;
 }
 
+// Chunk gather, part (b): dimension slice c of the text partials of the
+// score splits, merged (c < nm) into mt_o / mt_st.
+template <int D, int GM, int NTHR>
+__device__ void gather_text_slice(const StepParams& p, int c, int64_t hrow0, float (*tw)[kNsMax], float (*tl)[kNsMax]) {
+  constexpr int D4 = D / 4;
+  const int tid = threadIdx.x, G = p.G, ns = p.ns;
+  for (int i = tid; i < G * ns; i += NTHR) {
+    const int h = i / ns, s = i % ns;
+    const float2 r = __ldcg(reinterpret_cast<const float2*>(p.split_st + ((hrow0 + h) * p.nsp_max + s) * ST_N));
+    tw[h][s] = r.x;  // ST_MT
+    tl[h][s] = r.y;  // ST_L1T
+  }
+  __syncthreads();
+  if (tid < G) {
+    const int h = tid;
+    float M = -CUDART_INF_F;
+    for (int s = 0; s < ns; ++s) M = fmaxf(M, tw[h][s]);
+    float L = 0.f;
+    for (int s = 0; s < ns; ++s) {
+      const float w = exp2_rel(tw[h][s], M);
+      tw[h][s] = w;
+      L = fmaf(w, tl[h][s], L);
+    }
+    if (c == 0) {
+      p.mt_st[(hrow0 + h) * 2 + 0] = M;
+      p.mt_st[(hrow0 + h) * 2 + 1] = L;
+    }
+  }
+  __syncthreads();
+  const int s4 = D4 / p.nm;  // float4s of this CTA's slice, per head
+  for (int i = tid; i < G * s4; i += NTHR) {
+    const int h = i / s4, d = 4 * (c * s4 + i % s4);
+    const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
+    float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+    for (int s = 0; s < ns; ++s) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
+      const float w = tw[h][s];
+      num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
+    }
+    *reinterpret_cast<float4*>(p.mt_o + (hrow0 + h) * D + d) = num;
+  }
+}
+
+// Chunk gather, finish: the last CTA of (sequence, kv-head) to arrive combines
+// the text output with the kept chunks (log-sum-exp form) and writes out.
+// The text part is the merged slice output, or the single split partial.
+template <typename T, int D, int GM, int NTHR>
+__device__ void gather_finish(const StepParams& p, int b, int g, int64_t hrow0, int64_t pbase,
+                              float (*tw)[kNsMax], float (*fin)[4], int* last) {
+  constexpr int D4 = D / 4;
+  const int tid = threadIdx.x, G = p.G;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) *last = atomicAdd(p.tickets + (int64_t)b * p.Hkv + g, 1u) == (unsigned)p.nc - 1u;
+  __syncthreads();
+  if (!*last) return;
+  __threadfence();
+  const float* t_o = p.nm ? p.mt_o + hrow0 * D : p.split_o + hrow0 * p.nsp_max * D;
+  const int t_ostride = p.nm ? D : p.nsp_max * D;
+  if (tid < G) {
+    const int h = tid;
+    float mt, lt;
+    if (p.nm) {
+      mt = __ldcg(p.mt_st + (hrow0 + h) * 2);
+      lt = __ldcg(p.mt_st + (hrow0 + h) * 2 + 1);
+    } else {
+      mt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_MT);
+      lt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_L1T);
+    }
+    float M = mt;
+    for (int k = 0; k < p.nk; ++k) M = fmaxf(M, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2));
+    const float wt = exp2_rel(mt, M);
+    float den = wt * lt;
+    for (int k = 0; k < p.nk; ++k) {
+      const float w = exp2_rel(__ldcg(p.gpart_st + ((pbase + k) * G + h) * 2), M);
+      tw[h][k] = w;
+      den = fmaf(w, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2 + 1), den);
+    }
+    fin[h][0] = wt;
+    fin[h][1] = den > 0.f ? 1.f / den : 0.f;
+  }
+  __syncthreads();
+  for (int i = tid; i < G * D4; i += NTHR) {
+    const int h = i / D4, d = 4 * (i % D4);
+    const float wt = fin[h][0];
+    const float4 tv = __ldcg(reinterpret_cast<const float4*>(t_o + (int64_t)h * t_ostride + d));
+    float4 num = make_float4(wt * tv.x, wt * tv.y, wt * tv.z, wt * tv.w);
+#pragma unroll 4
+    for (int k = 0; k < p.nk; ++k) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(p.gpart_o + ((pbase + k) * G + h) * D + d));
+      const float w = tw[h][k];
+      num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
+    }
+    const float inv = fin[h][1];
+    T* o = reinterpret_cast<T*>(p.out) + (hrow0 + h) * D + d;
+    o[0] = from_f<T>(num.x * inv); o[1] = from_f<T>(num.y * inv);
+    o[2] = from_f<T>(num.z * inv); o[3] = from_f<T>(num.w * inv);
+  }
+  if (tid == 0) p.tickets[(int64_t)b * p.Hkv + g] = 0u;
+}
+
 // ---------------------------------------------------------------------------
 // k_gather: grid (nc, Hkv, B), 256 threads.  CTA c (a) attends over chunk c of
 // the kept list (c < nk), staged 64 tokens at a time -- indices, V-row
@@ -1521,7 +1639,6 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
   constexpr int CH = 16 / sizeof(T);          // elements per 16-byte slice
   constexpr int CPR = D / CH;                 // slices per row
   constexpr int SLOTS = kGatherThreads / CPR; // tokens processed side by side
-  constexpr int D4 = D / 4;
   static_assert(kGatherThreads % CPR == 0 && CPR <= 32, "row slicing");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   auto& sm = *reinterpret_cast<GatherSmem<T, D, GM>*>(smem_raw);
@@ -1653,99 +1770,271 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
     }
   }
 
-  // (b) dimension slice c of the text partials
-  if (c < p.nm) {
-    const int ns = p.ns;
-    for (int i = tid; i < G * ns; i += kGatherThreads) {
-      const int h = i / ns, s = i % ns;
-      const float2 r = __ldcg(reinterpret_cast<const float2*>(p.split_st + ((hrow0 + h) * p.nsp_max + s) * ST_N));
-      sm.tw[h][s] = r.x;  // ST_MT
-      sm.tl[h][s] = r.y;  // ST_L1T
-    }
-    __syncthreads();
-    if (tid < G) {
-      const int h = tid;
-      float M = -CUDART_INF_F;
-      for (int s = 0; s < ns; ++s) M = fmaxf(M, sm.tw[h][s]);
-      float L = 0.f;
-      for (int s = 0; s < ns; ++s) {
-        const float w = exp2_rel(sm.tw[h][s], M);
-        sm.tw[h][s] = w;
-        L = fmaf(w, sm.tl[h][s], L);
-      }
-      if (c == 0) {
-        p.mt_st[(hrow0 + h) * 2 + 0] = M;
-        p.mt_st[(hrow0 + h) * 2 + 1] = L;
-      }
-    }
-    __syncthreads();
-    const int s4 = D4 / p.nm;  // float4s of this CTA's slice, per head
-    for (int i = tid; i < G * s4; i += kGatherThreads) {
-      const int h = i / s4, d = 4 * (c * s4 + i % s4);
-      const float* so = p.split_o + (hrow0 + h) * p.nsp_max * D + d;
-      float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-      for (int s = 0; s < ns; ++s) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(so + (int64_t)s * D));
-        const float w = sm.tw[h][s];
-        num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
-      }
-      *reinterpret_cast<float4*>(p.mt_o + (hrow0 + h) * D + d) = num;
-    }
-  }
+  if (c < p.nm) gather_text_slice<D, GM, kGatherThreads>(p, c, hrow0, sm.tw, sm.tl);
   if (err) atomicOr(p.err, err);
+  gather_finish<T, D, GM, kGatherThreads>(p, b, g, hrow0, pbase, sm.tw, sm.fin, &sm.last);
+}
 
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) sm.last = atomicAdd(p.tickets + (int64_t)b * p.Hkv + g, 1u) == (unsigned)p.nc - 1u;
-  __syncthreads();
-  if (!sm.last) return;
-  __threadfence();
+// ---------------------------------------------------------------------------
+// k_gather_mma (bf16): grid (nc, Hkv, B), 4 warps.  CTA c (a) attends over
+// chunk c of the kept list (c < nk).  Warp w takes 32-token tiles w, w + 4,
+// ... of the chunk and streams the kept V rows through a private ring of
+// three slots: lane t bulk-copies row t of a tile into a row padded to
+// 2D + 16 bytes (conflict-free ldmatrix), after lane 0 armed the slot's
+// mbarrier with the tile's byte count.  The tile's logits (read one tile
+// ahead) give per-head running maxima and probabilities; P.V runs on the
+// tensor cores as in the score kernel (A = V^T by ldmatrix.trans, B = P^T
+// from a per-warp bf16 buffer).  The warps' partials are merged into the
+// chunk's partial; (b) and the final combine are shared with k_gather.
+// ---------------------------------------------------------------------------
+constexpr int kGmWarps = 4;
+constexpr int kGmSlots = 3;
+constexpr int kGmMaxChunk = 1024;  // kept rows per CTA (the plan's chunks are at most this)
 
-  // Last CTA: combine the text output with the kept chunks (log-sum-exp form).
-  // The text part is the merged slice output, or the single split partial.
-  const float* t_o = p.nm ? p.mt_o + hrow0 * D : p.split_o + hrow0 * p.nsp_max * D;
-  const int t_ostride = p.nm ? D : p.nsp_max * D;
-  if (tid < G) {
-    const int h = tid;
-    float mt, lt;
-    if (p.nm) {
-      mt = __ldcg(p.mt_st + (hrow0 + h) * 2);
-      lt = __ldcg(p.mt_st + (hrow0 + h) * 2 + 1);
-    } else {
-      mt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_MT);
-      lt = __ldcg(p.split_st + (hrow0 + h) * p.nsp_max * ST_N + ST_L1T);
-    }
-    float M = mt;
-    for (int k = 0; k < p.nk; ++k) M = fmaxf(M, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2));
-    const float wt = exp2_rel(mt, M);
-    float den = wt * lt;
-    for (int k = 0; k < p.nk; ++k) {
-      const float w = exp2_rel(__ldcg(p.gpart_st + ((pbase + k) * G + h) * 2), M);
-      sm.tw[h][k] = w;
-      den = fmaf(w, __ldcg(p.gpart_st + ((pbase + k) * G + h) * 2 + 1), den);
-    }
-    sm.fin[h][0] = wt;
-    sm.fin[h][1] = den > 0.f ? 1.f / den : 0.f;
-  }
+template <int D, int NT>
+struct GmCfg {
+  static constexpr int GM = 8 * NT;
+  static constexpr int THREADS = 32 * kGmWarps;
+  static constexpr int MT = D / 16;
+  static constexpr int HALF_BYTES = 32 * 128;                   // 32 rows x 64 dimensions
+  static constexpr int SLOT = (D / 64) * HALF_BYTES;            // 32 V rows, swizzled
+  static constexpr int RING = kGmWarps * kGmSlots * SLOT;
+  static constexpr int OFF_BAR = RING;                          // full[warps][slots]
+  // Logits of a slot's tokens, float [GM][32]; once read, the tile's bf16
+  // probabilities [GM][32] take their place.
+  static constexpr int OFF_Z = OFF_BAR + kGmWarps * kGmSlots * 8;
+  static constexpr int OFF_MASK = OFF_Z + kGmWarps * kGmSlots * GM * 32 * 4;   // copied rows per slot
+  static constexpr int OFF_WST = OFF_MASK + kGmWarps * kGmSlots * 4;          // float [warps][GM][2]
+  static constexpr int OFF_FIN = OFF_WST + kGmWarps * GM * 2 * 4;             // float [GM][4]
+  static constexpr int OFF_LAST = OFF_FIN + GM * 4 * 4;
+  static constexpr int OFF_KIDX = OFF_LAST + 16;                // int16 [kGmMaxChunk] kept indices
+  static constexpr size_t SMEM = (size_t)OFF_KIDX + kGmMaxChunk * 2;
+  // After part (a) the ring holds the warps' outputs, then the split weights.
+  static constexpr int OFF_TW = kGmWarps * GM * D * 4;
+  static_assert(OFF_TW + 2 * GM * kNsMax * 4 <= RING, "reuse of the ring");
+  static_assert(OFF_Z % 16 == 0 && OFF_WST % 16 == 0, "alignment");
+};
+
+template <int D, int NT>
+__global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_constant__ StepParams p) {
+  using C = GmCfg<D, NT>;
+  constexpr int GM = C::GM, S = kGmSlots;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  unsigned char* smem = smem_raw;
+  const int c = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gr = lane >> 2, tg = lane & 3;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + warp * S;
+  float* zs = reinterpret_cast<float*>(smem + C::OFF_Z) + warp * S * GM * 32;
+  uint32_t* mask_s = reinterpret_cast<uint32_t*>(smem + C::OFF_MASK) + warp * S;
+  float (*wst)[GM][2] = reinterpret_cast<float (*)[GM][2]>(smem + C::OFF_WST);
+  float (*fin)[4] = reinterpret_cast<float (*)[4]>(smem + C::OFF_FIN);
+  int* last = reinterpret_cast<int*>(smem + C::OFF_LAST);
+  short* kidx = reinterpret_cast<short*>(smem + C::OFF_KIDX);  // indices < 32768
+  unsigned char* ring = smem + warp * S * C::SLOT;
+
+  // A slot's phase completes when all 32 lanes' copies have landed.
+  if (tid < kGmWarps * S) mbar_init(reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + tid, 32);
+  mbar_fence_init();
   __syncthreads();
-  for (int i = tid; i < G * D4; i += kGatherThreads) {
-    const int h = i / D4, d = 4 * (i % D4);
-    const float wt = sm.fin[h][0];
-    const float4 tv = __ldcg(reinterpret_cast<const float4*>(t_o + (int64_t)h * t_ostride + d));
-    float4 num = make_float4(wt * tv.x, wt * tv.y, wt * tv.z, wt * tv.w);
-#pragma unroll 4
-    for (int k = 0; k < p.nk; ++k) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(p.gpart_o + ((pbase + k) * G + h) * D + d));
-      const float w = sm.tw[h][k];
-      num.x = fmaf(w, v.x, num.x); num.y = fmaf(w, v.y, num.y); num.z = fmaf(w, v.z, num.z); num.w = fmaf(w, v.w, num.w);
-    }
-    const float inv = sm.fin[h][1];
-    T* o = reinterpret_cast<T*>(p.out) + (hrow0 + h) * D + d;
-    o[0] = from_f<T>(num.x * inv); o[1] = from_f<T>(num.y * inv);
-    o[2] = from_f<T>(num.z * inv); o[3] = from_f<T>(num.w * inv);
+  const int G = p.G, H = p.H;
+  const int64_t hrow0 = (int64_t)b * H + g * G;
+  float (*tw)[kNsMax] = reinterpret_cast<float (*)[kNsMax]>(smem + C::OFF_TW);
+  float (*tl)[kNsMax] = tw + GM;
+  // (b) first: it reads only the score kernel's partials, complete before the
+  // select kernel lets this grid start.  Its shared memory is the ring's.
+  if (c < p.nm) {
+    gather_text_slice<D, GM, C::THREADS>(p, c, hrow0, tw, tl);
+    fence_proxy_async();
+    __syncthreads();
   }
-  if (tid == 0) p.tickets[(int64_t)b * p.Hkv + g] = 0u;
+  pdl_wait();
+  pdl_trigger();
+  const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
+  unsigned err = 0;
+  bool timed_out = false;
+
+  // (a) kept chunk c
+  if (c < p.nk) {
+    const Seq sq = load_seq(p, b, false);
+    const int sel = p.granularity ? b * p.Hkv + g : b;
+    const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
+    const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
+    const int per = (K + p.nk - 1) / p.nk;
+    const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + kGmMaxChunk));
+    if (per > kGmMaxChunk) err |= ERR_KEPT;  // the plan keeps every chunk within the limit
+    // The chunk's kept indices, read once (out-of-range ones become -1).
+    for (int j = j0 + tid; j < j1; j += C::THREADS) {
+      int i = __ldg(kept + j);
+      if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
+      kidx[j - j0] = (short)i;
+    }
+    const int ntile = (j1 - j0 + 31) / 32;
+    const int nj = warp < ntile ? (ntile - warp + kGmWarps - 1) / kGmWarps : 0;  // this warp's tiles
+    const float* zb = p.z_ws + (int64_t)b * p.max_visual * p.hp + g * G;
+    int issued = 0;  // tiles of this warp whose copies were issued
+    __syncthreads();
+
+    // Kept index of row `lane` of this warp's tile k, or -1.
+    auto row_index = [&](int k) {
+      const int j = 32 * (warp + kGmWarps * k) + lane;
+      return (k < nj && j0 + j < j1) ? (int)kidx[j] : -1;
+    };
+    auto issue = [&](int k, int i) {  // all lanes; i = this lane's kept index
+      if (k >= nj) return;
+      const int slot = k % S;
+      const __nv_bfloat16* vr = nullptr;
+      if (i >= 0) {
+        vr = kv_row<__nv_bfloat16>(p.v, p, b, g, sq.vs + i);
+        if (!vr) { err |= ERR_PAGE; i = -1; }
+      }
+      const unsigned m = __ballot_sync(0xffffffffu, vr != nullptr);
+      if (lane == 0) mask_s[slot] = m;
+      __syncwarp();  // every lane is done reading this slot
+      // V rows: instruction j copies piece (lane % PPR) of row j * RPI + lane / PPR.
+      constexpr int PPR = 2 * D / 16, RPI = 32 / PPR;
+      const unsigned sbase = smem_u32(ring + slot * C::SLOT);
+      const unsigned long long src = reinterpret_cast<unsigned long long>(vr);
+#pragma unroll
+      for (int j = 0; j < 32 / RPI; ++j) {
+        const int row = j * RPI + lane / PPR;
+        const unsigned long long r = __shfl_sync(0xffffffffu, src, row);
+        if (r) cp_async16(sbase + swz_off<C::HALF_BYTES>(row, 8 * (lane % PPR)),
+                          reinterpret_cast<const char*>(r) + (lane % PPR) * 16);
+      }
+      // Logits of this lane's token.
+      if (vr) {
+        const float* zr = zb + (int64_t)i * p.hp;
+        const unsigned zd = smem_u32(zs + slot * GM * 32 + lane);
+        for (int h = 0; h < G; ++h) cp_async4(zd + h * 32 * 4, zr + h);
+      }
+      cp_async_arrive(full + slot);
+      issued = k + 1;
+    };
+    // Prologue: the first S tiles, each next row index already in flight.
+    int inext = row_index(0);
+#pragma unroll 1
+    for (int k = 0; k < S; ++k) {
+      const int icur = inext;
+      inext = row_index(k + 1);
+      issue(k, icur);
+    }
+    int ipend = inext;  // kept index for tile S (issued once tile 0 is read)
+
+    // Probabilities are taken relative to each head's largest logit over all
+    // tokens (from the select kernel), so no running maximum is needed.
+    float mh[GM], lsum[GM];
+    float acc[NT][C::MT][4];
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      mh[h] = h < G ? __ldcg(p.hmax + hrow0 + h) : -CUDART_INF_F;
+      lsum[h] = 0.f;
+    }
+#pragma unroll
+    for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+      for (int mi = 0; mi < C::MT; ++mi)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[nn][mi][e] = 0.f;
+    // ldmatrix.trans lane roles for V^T (A operand, rows = dimensions).
+    const int vrow = (lane & 7) + 8 * (lane >> 4), vcol = 8 * ((lane >> 3) & 1);
+
+    for (int k = 0; k < nj; ++k) {
+      const int slot = k % S;
+      if (!mbar_wait(full + slot, (k / S) & 1)) { timed_out = true; break; }
+      const uint32_t mask = mask_s[slot];
+      const bool live = (mask >> lane) & 1u;
+      float z[GM];
+#pragma unroll
+      for (int h = 0; h < GM; ++h) z[h] = (live && h < G) ? zs[(slot * GM + h) * 32 + lane] : -CUDART_INF_F;
+
+      // Probabilities of this tile, written over its logits.
+      __syncwarp();
+      __nv_bfloat16* P = reinterpret_cast<__nv_bfloat16*>(zs + slot * GM * 32);
+#pragma unroll
+      for (int h = 0; h < GM; ++h) {
+        if (h >= G) continue;
+        const float pe = exp2_rel(z[h], mh[h]);
+        lsum[h] += pe;
+        P[h * 32 + lane] = __float2bfloat16_rn(pe);
+      }
+      __syncwarp();
+      const unsigned vt = smem_u32(ring + slot * C::SLOT);
+#pragma unroll
+      for (int sb = 0; sb < 2; ++sb) {
+        uint32_t pb[NT][2];
+#pragma unroll
+        for (int nn = 0; nn < NT; ++nn) {
+          const __nv_bfloat16* pr = P + (8 * nn + gr) * 32 + 16 * sb + 2 * tg;
+          pb[nn][0] = *reinterpret_cast<const uint32_t*>(pr);
+          pb[nn][1] = *reinterpret_cast<const uint32_t*>(pr + 8);
+        }
+        // Rows that were not copied hold stale bytes: zero their words.  (B
+        // columns of heads past G hold stale bytes too; those heads' sums
+        // are never read.)
+        const uint32_t rb = mask >> (16 * sb);
+        const uint32_t mlo = (((rb >> (2 * tg)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 1)) & 1u) ? 0xffff0000u : 0u);
+        const uint32_t mhi = (((rb >> (2 * tg + 8)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 9)) & 1u) ? 0xffff0000u : 0u);
+#pragma unroll
+        for (int mi = 0; mi < C::MT; ++mi) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_t(vt + swz_off<C::HALF_BYTES>(16 * sb + vrow, 16 * mi + vcol), a0, a1, a2, a3);
+          a0 &= mlo; a1 &= mlo; a2 &= mhi; a3 &= mhi;
+#pragma unroll
+          for (int nn = 0; nn < NT; ++nn) mma_bf16(acc[nn][mi], a0, a1, a2, a3, pb[nn][0], pb[nn][1]);
+        }
+      }
+      __syncwarp();
+      // Refill this slot with tile k + S.
+      const int icur = ipend;
+      ipend = row_index(k + S + 1);
+      issue(k + S, icur);
+    }
+    // After a timeout, let this warp's copies still in flight land (bounded)
+    // before the ring is reused below.
+    if (timed_out && lane == 0)
+      for (int k = max(0, issued - S); k < issued; ++k) mbar_wait(full + k % S, (k / S) & 1);
+    __syncwarp();
+
+    // Warp partials -> chunk partial (log-sum-exp over the warps).
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      const float l = warp_sum(lsum[h]);
+      if (lane == 0) { wst[warp][h][0] = mh[h]; wst[warp][h][1] = l; }
+    }
+    __syncthreads();  // every warp is done with its ring
+    float* ow = reinterpret_cast<float*>(smem) + warp * GM * D;
+#pragma unroll
+    for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+      for (int mi = 0; mi < C::MT; ++mi) {
+        const int h0 = 8 * nn + 2 * tg, d0 = 16 * mi + gr;
+        ow[h0 * D + d0] = acc[nn][mi][0];
+        ow[(h0 + 1) * D + d0] = acc[nn][mi][1];
+        ow[h0 * D + d0 + 8] = acc[nn][mi][2];
+        ow[(h0 + 1) * D + d0 + 8] = acc[nn][mi][3];
+      }
+    __syncthreads();
+    for (int i = tid; i < G * D; i += C::THREADS) {
+      const int h = i / D, d = i % D;
+      float o = 0.f, l = 0.f;
+#pragma unroll
+      for (int w = 0; w < kGmWarps; ++w) {
+        o += reinterpret_cast<const float*>(smem)[(w * GM + h) * D + d];
+        l += wst[w][h][1];
+      }
+      p.gpart_o[((pbase + c) * G + h) * D + d] = o;
+      if (d == 0) {
+        p.gpart_st[((pbase + c) * G + h) * 2 + 0] = wst[0][h][0];
+        p.gpart_st[((pbase + c) * G + h) * 2 + 1] = l;
+      }
+    }
+    __syncthreads();  // the ring is reused below
+  }
+
+  if (timed_out) err |= ERR_TIMEOUT;
+  if (err) atomicOr(p.err, err);
+  gather_finish<__nv_bfloat16, D, GM, C::THREADS>(p, b, g, hrow0, pbase, tw, fin, last);
 }
 
 // ---------------------------------------------------------------------------
@@ -2012,6 +2301,10 @@ cudaError_t launch_gather_td(const StepParams& p, cudaStream_t st) {
     return launch_ex(k_gather_slice<T, D, 16>, grid, dim3(kGatherThreads), slice_smem<16>(), st, 1, p);
   }
   const dim3 grid(p.nc, p.Hkv, p.B);
+  if (sizeof(T) == 2) {
+    if (p.G <= 8) return launch_ex(k_gather_mma<D, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 1>::SMEM, st, 1, p);
+    return launch_ex(k_gather_mma<D, 2>, grid, dim3(32 * kGmWarps), GmCfg<D, 2>::SMEM, st, 1, p);
+  }
   if (p.G <= 4) return launch_ex(k_gather<T, D, 4>, grid, dim3(kGatherThreads), gather_smem<T, D, 4>(), st, 1, p);
   if (p.G <= 8) return launch_ex(k_gather<T, D, 8>, grid, dim3(kGatherThreads), gather_smem<T, D, 8>(), st, 1, p);
   return launch_ex(k_gather<T, D, 16>, grid, dim3(kGatherThreads), gather_smem<T, D, 16>(), st, 1, p);
@@ -2025,6 +2318,10 @@ cudaError_t set_smem(void (*kernel)(StepParams), size_t bytes) {
 cudaError_t configure_fixed_kernels() {
   cudaError_t e = cudaSuccess;
 #define VP_SET(kernel, bytes) if (e == cudaSuccess) e = set_smem(kernel, bytes)
+  VP_SET((k_gather_mma<128, 1>), (GmCfg<128, 1>::SMEM));
+  VP_SET((k_gather_mma<128, 2>), (GmCfg<128, 2>::SMEM));
+  VP_SET((k_gather_mma<64, 1>), (GmCfg<64, 1>::SMEM));
+  VP_SET((k_gather_mma<64, 2>), (GmCfg<64, 2>::SMEM));
   VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 1>()));
   VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 2>()));
   VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>()>), (tma_smem<64, 1>()));

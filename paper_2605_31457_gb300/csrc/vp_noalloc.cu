@@ -174,6 +174,7 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   p.gpart_st = reinterpret_cast<float*>(base + L.o_gs);
   p.mt_o = reinterpret_cast<float*>(base + L.o_mo);
   p.mt_st = reinterpret_cast<float*>(base + L.o_ms);
+  p.hmax = reinterpret_cast<float*>(base + L.o_hm);
   const vp::Plan pl = vp::make_plan(batch, Hkv, D, slot->num_sms, c.max_visual, c.max_seq, kept_cap,
                                     budget->granularity);
   p.hp = L.hp;
