@@ -123,8 +123,18 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   if (nk < nk_want) nk = nk_want < nk_small ? nk_want : nk_small;
   if (nk < 1) nk = 1;
   if (nk > kNkMax) nk = kNkMax;
-  const int nm = ns > 1 ? (D / 16 < kMaxMerge ? D / 16 : kMaxMerge) : 0;
-  return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), kept_cap <= 256 ? 1 : 0};
+  // Text-partial merge slices: as many as there are kept chunks (a power of
+  // two up to D / 16 and kMaxMerge), so that no CTA merges text alone.
+  int nm = 0;
+  if (ns > 1) {
+    const long long cap_m = D / 16 < kMaxMerge ? D / 16 : kMaxMerge;
+    nm = 1;
+    while (2LL * nm <= cap_m && 2LL * nm <= nk) nm *= 2;
+  }
+  // Small kept sets of few sequences: one CTA per 16 output dimensions, so
+  // that the whole gather is one short wave; otherwise one CTA per chunk.
+  const int gslice = kept_cap <= 256 && units * (D / 16) <= slots ? 1 : 0;
+  return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), gslice};
 }
 
 // Workspace layout for up to `batch` sequences (offsets in bytes, 256-aligned).

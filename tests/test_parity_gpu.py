@@ -117,6 +117,29 @@ def test_paged_bf16_page_sizes(vp, page_size, layout):
     Hn.check_all(vp, Hn.make_inputs(r), r.budget, layout=layout)
 
 
+def _many(batch, **kw):
+    """`batch` sequences with varied lengths (seeded), for the per-chunk gather."""
+    rng = np.random.default_rng(batch)
+    vis = tuple(int(x) for x in rng.integers(64, 700, batch))
+    start = tuple(int(x) for x in rng.integers(0, 40, batch))
+    text = tuple(int(s) + int(x) for s, x in zip(start, rng.integers(1, 300, batch)))
+    return small(batch=batch, vis_len=vis, vis_start=start, text_len=text, **kw)
+
+
+@pytest.mark.parametrize("dtype,D,batch,budget", [
+    (W.FP32, 64, 3, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000)),
+    (W.FP32, 128, 3, dict(mode=O.DENSE, tau=0.1)),
+    (W.BF16, 128, 40, W.ADAPTIVE_5PCT),
+    (W.BF16, 64, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000)),
+    (W.BF16, 128, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000, granularity=1)),
+])
+def test_chunk_gather_paths(vp, dtype, D, batch, budget):
+    """Kept sets above 256 rows (fp32 and bf16 chunk kernels), and many
+    sequences with small kept sets, which also take the chunk kernel."""
+    r = _many(batch, dtype=dtype, head_dim=D) if batch > 3 else small(dtype=dtype, head_dim=D)
+    Hn.check_all(vp, Hn.make_inputs(r), budget)
+
+
 def test_explicit_logit_scale(vp):
     r = small()
     Hn.check_all(vp, Hn.make_inputs(r), dict(r.budget, scale=0.05))
