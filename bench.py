@@ -49,6 +49,9 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU-baseline leg")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline sample budget")
+    ap.add_argument("--layer-calls", type=int, default=0,
+                    help="profiling aid: N calls on one layer of the workload, no timing")
+    ap.add_argument("--flush-l2", action="store_true", help="with --layer-calls: flush L2 before every call")
     return ap.parse_args(argv)
 
 
@@ -452,42 +455,61 @@ def run_ours(args, rank, world, local):
 
 
 def e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, world):
-    """Same steps through the C ABI with host buffers: every step copies its
-    queries and the appended token's K/V in from pinned memory, runs the 28
-    layer calls and copies the outputs, kept sets, budgets and masses back."""
+    """Same steps through the C ABI, fed from and read back to host memory, as
+    a serving loop drives it: every step copies its queries, the appended
+    token's K/V of every layer and the text lengths in from pinned memory
+    (three copies into staging buffers), replays that step's CUDA graph -- the
+    appends into the caches and the 28 vp_decode_step calls, captured once
+    through the C ABI -- and copies the outputs, kept sets, budgets and masses
+    back, with one stream synchronisation per step."""
     import torch
-    L, B, H, D = r.layers, r.batch, r.heads, r.head_dim
+    L, B, H, D, Hkv = r.layers, r.batch, r.heads, r.head_dim, r.kv_heads
     S = args.warmup + args.steps
     nv0, tl0 = int(r.vis_lens[0]), int(r.text_lens[0])
-    qh = q_host.pin_memory()
-    newk = torch.stack([k[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for k in ks]).cpu().pin_memory()
-    newv = torch.stack([v[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for v in vs_]).cpu().pin_memory()
+    qh = q_host.pin_memory()                                           # [S, L, B, H, D]
+    kvh = torch.stack([torch.stack([k[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for k in ks]),
+                       torch.stack([v[:, :, nv0 + tl0 - 1: nv0 + tl0 - 1 + S] for v in vs_])])
+    kvh = kvh.permute(4, 0, 1, 2, 3, 5).contiguous().cpu().pin_memory()   # [S, 2, L, B, Hkv, D]
+    tlh = (torch.tensor(r.text_lens, dtype=torch.int32)[None, :] + torch.arange(S, dtype=torch.int32)[:, None]
+           ).contiguous().pin_memory()                                  # [S, B]
     q_in = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
+    kv_in = torch.empty((2, L, B, Hkv, D), dtype=torch.bfloat16, device=dev)
     tl = torch.empty((B,), dtype=torch.int32, device=dev)
-    tl_host = torch.empty((B,), dtype=torch.int32).pin_memory()
     out = torch.empty((L, B, H, D), dtype=torch.bfloat16, device=dev)
     kept = torch.empty((L, B, cap), dtype=torch.int32, device=dev)
     count = torch.empty((L, B), dtype=torch.int32, device=dev)
     mass = torch.empty((L, B, H), dtype=torch.float32, device=dev)
     stats = torch.empty((L, B, 4), dtype=torch.float32, device=dev)
     res = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (out, kept, count, mass, stats)]
-    stream = torch.cuda.current_stream()
+    stream = torch.cuda.Stream(device=dev)
 
-    def one(s):
+    def calls(s):
         pos = nv0 + tl0 - 1 + s
-        tl_host.fill_(tl0 + s)
-        tl.copy_(tl_host, non_blocking=True)
-        q_in.copy_(qh[s], non_blocking=True)
         for layer in range(L):
-            ks[layer][:, :, pos].copy_(newk[layer][:, :, s], non_blocking=True)
-            vs_[layer][:, :, pos].copy_(newv[layer][:, :, s], non_blocking=True)
+            ks[layer][:, :, pos].copy_(kv_in[0, layer])
+            vs_[layer][:, :, pos].copy_(kv_in[1, layer])
             vp.vp_decode_step(ctx, B, q_in[layer], kc[layer], vc[layer], span, tl, budget, out[layer],
                               kept[layer], cap, count[layer], mass[layer], stats[layer], stream=stream)
-        for dst, src in zip(res, (out, kept, count, mass, stats)):
-            dst.copy_(src, non_blocking=True)
-        stream.synchronize()
 
     vp.vp_timing_enable(ctx, 0)
+    graphs = []
+    for s in range(S):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            calls(s)
+        graphs.append(g)
+    torch.cuda.synchronize()
+
+    def one(s):
+        with torch.cuda.stream(stream):
+            q_in.copy_(qh[s], non_blocking=True)
+            kv_in.copy_(kvh[s], non_blocking=True)
+            tl.copy_(tlh[s], non_blocking=True)
+            graphs[s].replay()
+            for dst, src in zip(res, (out, kept, count, mass, stats)):
+                dst.copy_(src, non_blocking=True)
+        stream.synchronize()
+
     for s in range(args.warmup):
         one(s)
     torch.cuda.synchronize()
@@ -501,12 +523,61 @@ def e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, w
         t = torch.tensor([el], dtype=torch.float64, device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         el = float(t.item())
-    esz = 2
-    h2d = 4 * B + L * B * H * D * esz + 2 * L * B * r.kv_heads * D * esz
+    h2d = sum(t[0].numel() * t.element_size() for t in (qh, kvh, tlh))
     d2h = sum(t.numel() * t.element_size() for t in (out, kept, count, mass, stats))
     return {"value": world * args.steps / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": el * 1e3 / args.steps,
-            "note": "direct C-ABI calls (no graph), host wall clock, one stream sync per step"}
+            "note": "host wall clock per step: pinned-host inputs copied in, the step's CUDA graph (K/V appends "
+                    "+ 28 vp_decode_step calls captured through the C ABI) replayed, results copied back, "
+                    "one stream sync per step"}
+
+
+def run_layer_calls(args):
+    """--layer-calls N: one layer of the workload, N back-to-back calls and a
+    device check, for profiling a single launch of each kernel (optionally
+    with the L2 flushed by a 256 MB write before every call)."""
+    import torch
+    from paper_2605_31457_gb300 import vp, workloads as W
+    r, _, _, _ = pick_workload(args.workload)
+    dev = torch.device("cuda")
+    B, H, Hkv, D = r.batch, r.heads, r.kv_heads, r.head_dim
+    t_cap = r.capacity(2)
+    k, v, f, sk = W.make_layer_torch(r, 0, t_cap, dev)
+    q = W.make_queries_torch(r, 0, 1, f, sk, dev)[0]
+    if r.paged:
+        bt_np, n_pages, _ = W.page_table(B, t_cap, r.page_size, r.seed)
+        bt = torch.from_numpy(bt_np).to(dev)
+        k = W.scatter_pages(k, bt_np, n_pages, r.page_size)
+        v = W.scatter_pages(v, bt_np, n_pages, r.page_size)
+        kc, vc = vp.kv_paged(k, bt), vp.kv_paged(v, bt)
+    else:
+        kc, vc = vp.kv_contiguous(k), vp.kv_contiguous(v)
+    vs = torch.tensor(r.vis_starts, dtype=torch.int32, device=dev)
+    vl = torch.tensor(r.vis_lens, dtype=torch.int32, device=dev)
+    tl = torch.tensor(r.text_lens, dtype=torch.int32, device=dev)
+    budget = vp.make_budget(**r.budget)
+    nvm = int(r.vis_lens.max())
+    cdt = torch.bfloat16 if r.dtype == W.BF16 else torch.float32
+    cfg = vp.make_config(B, H, Hkv, D, nvm, int((r.vis_lens + r.text_lens).max()) + 2,
+                         vp.VP_BF16 if r.dtype == W.BF16 else vp.VP_FP32, int(r.paged), r.page_size)
+    ctx = vp.vp_init(cfg)
+    cap = max(1, vp.vp_max_kept(budget, nvm))
+    out = torch.empty((B, H, D), dtype=cdt, device=dev)
+    kept = torch.empty((B, cap), dtype=torch.int32, device=dev)
+    cnt = torch.empty((B,), dtype=torch.int32, device=dev)
+    mass = torch.empty((B, H), dtype=torch.float32, device=dev)
+    st = torch.empty((B, 4), dtype=torch.float32, device=dev)
+    flush = torch.empty(64 << 20, dtype=torch.float32, device=dev) if args.flush_l2 else None
+    for _ in range(args.layer_calls):
+        if flush is not None:
+            flush.zero_()
+        vp.vp_decode_step(ctx, B, q, kc, vc, vp.span(vs, vl), tl, budget, out, kept, cap, cnt, mass, st)
+    torch.cuda.synchronize()
+    vp.vp_check_errors(ctx)
+    vp.vp_free(ctx)
+    print(json.dumps({"layer_calls": args.layer_calls, "workload": args.workload, "flush_l2": bool(args.flush_l2),
+                      "kv_bytes": 2 * k.numel() * k.element_size(), "avg_kept": float(cnt.float().mean())}))
+    return 0
 
 
 def committed_traffic():
@@ -529,6 +600,8 @@ def main(argv=None):
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.layer_calls:
+        return run_layer_calls(args)
     if world > 1:
         import torch
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
