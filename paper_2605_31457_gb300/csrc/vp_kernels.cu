@@ -660,6 +660,8 @@ __device__ __forceinline__ float fexp2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// exp2(a - m) by the hardware approximation, an empty term (a = -inf) giving 0.
+__device__ __forceinline__ float fexp2_rel(float a, float m) { return a == -CUDART_INF_F ? 0.f : fexp2(a - m); }
 __device__ __forceinline__ void tma_load_4d(unsigned dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
                                             uint64_t* bar) {
   asm volatile(
@@ -1251,14 +1253,14 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   constexpr int NW = NTH / 32;
   extern __shared__ __align__(16) uint32_t key_s[];  // [max_visual] score keys (rank 0's copy is used)
   __shared__ float hM_s[kMaxHeads], hInv_s[kMaxHeads], hMass_s[kMaxHeads], hMass1_s[kMaxHeads];
-  __shared__ unsigned hist_s[256];
+  __shared__ unsigned hist_s[3][256];  // one per radix pass, used in turn
   __shared__ int wsum_s[32];
   __shared__ int sh_i[4];
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
   const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int i = tid; i < 256; i += NTH) hist_s[i] = 0;
+  for (int i = tid; i < 3 * 256; i += NTH) (&hist_s[0][0])[i] = 0;
   pdl_wait();
   pdl_trigger();
   const int H = p.H, ns = p.ns;
@@ -1381,24 +1383,24 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
       for (int q = 0; q < 8; ++q) {
         if (4 * q < hcnt) {
           const int h = hbeg + 4 * q;
-          a = fmaf(exp2_rel(zpre[q].x, hM_s[h]), hInv_s[h], a);
-          a = fmaf(exp2_rel(zpre[q].y, hM_s[h + 1]), hInv_s[h + 1], a);
-          a = fmaf(exp2_rel(zpre[q].z, hM_s[h + 2]), hInv_s[h + 2], a);
-          a = fmaf(exp2_rel(zpre[q].w, hM_s[h + 3]), hInv_s[h + 3], a);
+          a = fmaf(fexp2_rel(zpre[q].x, hM_s[h]), hInv_s[h], a);
+          a = fmaf(fexp2_rel(zpre[q].y, hM_s[h + 1]), hInv_s[h + 1], a);
+          a = fmaf(fexp2_rel(zpre[q].z, hM_s[h + 2]), hInv_s[h + 2], a);
+          a = fmaf(fexp2_rel(zpre[q].w, hM_s[h + 3]), hInv_s[h + 3], a);
         }
       }
     } else if (vec) {
       for (int hh = 0; hh < hcnt; hh += 4) {
         const float4 z4 = __ldcg(reinterpret_cast<const float4*>(zr + hh));
         const int h = hbeg + hh;
-        a = fmaf(exp2_rel(z4.x, hM_s[h]), hInv_s[h], a);
-        a = fmaf(exp2_rel(z4.y, hM_s[h + 1]), hInv_s[h + 1], a);
-        a = fmaf(exp2_rel(z4.z, hM_s[h + 2]), hInv_s[h + 2], a);
-        a = fmaf(exp2_rel(z4.w, hM_s[h + 3]), hInv_s[h + 3], a);
+        a = fmaf(fexp2_rel(z4.x, hM_s[h]), hInv_s[h], a);
+        a = fmaf(fexp2_rel(z4.y, hM_s[h + 1]), hInv_s[h + 1], a);
+        a = fmaf(fexp2_rel(z4.z, hM_s[h + 2]), hInv_s[h + 2], a);
+        a = fmaf(fexp2_rel(z4.w, hM_s[h + 3]), hInv_s[h + 3], a);
       }
     } else {
       for (int hh = 0; hh < hcnt; ++hh)
-        a = fmaf(exp2_rel(__ldcg(zr + hh), hM_s[hbeg + hh]), hInv_s[hbeg + hh], a);
+        a = fmaf(fexp2_rel(__ldcg(zr + hh), hM_s[hbeg + hh]), hInv_s[hbeg + hh], a);
     }
     const float sc = a * inv_cnt;
     if (!isfinite(sc)) bad = 1;
@@ -1413,15 +1415,20 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
 
   // 4. Radix select of the K-th largest key, 8 bits per pass from the top;
-  //    lanes holding the same digit add to the histogram once per warp.  Warp
-  //    0 scans the histogram and clears it for the next pass.
+  //    lanes holding the same digit add to the histogram once per warp.  One
+  //    barrier per pass: every warp scans the finished histogram itself, and
+  //    pass p clears the buffer of pass p - 2 for pass p + 1.
   const bool take_all = K >= nv;
   uint32_t theta = 0;
   unsigned krem = 0, n_theta = 0;  // keys equal to theta: to keep, in total
   if (K > 0 && !take_all) {
     uint32_t prefix = 0, mask = 0;
     krem = (unsigned)K;
-    for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      unsigned* hist = hist_s[pass % 3];
+      if (pass >= 2)  // the buffer of pass - 2, scanned by every warp before the last barrier
+        for (int i = tid; i < 256; i += NTH) hist_s[(pass + 1) % 3][i] = 0;
       for (int base = 0; base < nv; base += NTH) {
         const int i = base + tid;
         const uint32_t k = i < nv ? key_s[i] : 0u;
@@ -1432,48 +1439,42 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
           const int leader = __ffs(act) - 1;
           const unsigned d0 = __shfl_sync(0xffffffffu, dg, leader);
           if (__all_sync(0xffffffffu, !m || dg == d0)) {
-            if (lane == leader) atomicAdd(&hist_s[d0], (unsigned)__popc(act));
+            if (lane == leader) atomicAdd(&hist[d0], (unsigned)__popc(act));
           } else if (m) {
-            atomicAdd(&hist_s[dg], 1u);
+            atomicAdd(&hist[dg], 1u);
           }
         }
       }
       __syncthreads();
-      if (warp == 0) {
-        // Lane L owns digits 255-8L ... 248-8L (descending).
-        unsigned c[8], tot = 0;
+      // Lane L owns digits 255-8L ... 248-8L (descending).
+      unsigned c[8], tot = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) { c[j] = hist[255 - 8 * lane - j]; tot += c[j]; }
+      unsigned incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      const unsigned excl = incl - tot;
+      const bool mine = excl < krem && krem <= incl;
+      unsigned dsel = 0, before = 0, cnt = 0;
+      if (mine) {
+        unsigned run = excl;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          c[j] = hist_s[255 - 8 * lane - j];
-          hist_s[255 - 8 * lane - j] = 0;
-          tot += c[j];
-        }
-        unsigned incl = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += n;
-        }
-        const unsigned excl = incl - tot;
-        if (excl < krem && krem <= incl) {
-          unsigned run = excl;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (run + c[j] >= krem) {
-              sh_i[1] = 255 - 8 * lane - j;
-              sh_i[2] = (int)run;
-              sh_i[3] = (int)c[j];
-              break;
-            }
-            run += c[j];
-          }
+          if (run + c[j] >= krem) { dsel = 255 - 8 * lane - j; before = run; cnt = c[j]; break; }
+          run += c[j];
         }
       }
-      __syncthreads();
-      krem -= (unsigned)sh_i[2];
-      prefix |= (uint32_t)sh_i[1] << shift;
+      const int src = max(__ffs(__ballot_sync(0xffffffffu, mine)) - 1, 0);
+      dsel = __shfl_sync(0xffffffffu, dsel, src);
+      before = __shfl_sync(0xffffffffu, before, src);
+      cnt = __shfl_sync(0xffffffffu, cnt, src);
+      krem -= before;
+      prefix |= dsel << shift;
       mask |= 255u << shift;
-      if (shift == 0) n_theta = (unsigned)sh_i[3];
+      if (shift == 0) n_theta = cnt;
     }
     theta = prefix;  // the K-th largest key; krem keys equal to it are kept
   }
@@ -1481,7 +1482,8 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   // 5. Ascending compaction: keys above theta, plus the first krem equal keys
   //    (every equal key when there is no tie to break: one scan less).
   if (K > 0) {
-    const int per_t = (nv + NTH - 1) / NTH;
+    // An odd chunk length keeps the threads' reads in distinct banks.
+    const int per_t = ((nv + NTH - 1) / NTH) | 1;
     const int j0 = min(nv, tid * per_t), j1 = min(nv, j0 + per_t);
     const bool ties = !take_all && krem < n_theta;
     int n_eq = 0;

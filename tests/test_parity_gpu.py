@@ -263,3 +263,61 @@ def test_sweep_points(vp, nv):
     inp = Hn.make_inputs(W.sweep_recipe(nv, W.ADAPTIVE_5PCT))
     for budget in W.SWEEP_BUDGETS:
         Hn.check_all(vp, inp, budget, seqs=(0, 31, 63))
+
+
+# ------------------------------------------------- full sizes, device-generated
+
+def _device_generated(vp, r, seqs, budgets, rep):
+    """One layer of `r` at full size, drawn by the benchmark's on-device
+    generator and run in the launch configuration the benchmark times; the
+    sampled sequences are copied to the host and checked against the oracle."""
+    dev = torch.device("cuda")
+    t_cap = r.capacity(1)
+    k, v, f, sk = W.make_layer_torch(r, 0, t_cap, dev)
+    q = W.make_queries_torch(r, 0, 1, f, sk, dev)[0]
+    B, H, Hkv, D = r.batch, r.heads, r.kv_heads, r.head_dim
+    nvs, tls, vss = r.vis_lens, r.text_lens, r.vis_starts
+    cfg = vp.make_config(B, H, Hkv, D, int(nvs.max()), int((nvs + tls).max()), vp.VP_BF16, 0, 1)
+    ctx = vp.vp_init(cfg)
+    vs_d = torch.from_numpy(vss.astype(np.int32)).to(dev)  # kept alive: the span holds raw pointers
+    vl_d = torch.from_numpy(nvs.astype(np.int32)).to(dev)
+    span = vp.span(vs_d, vl_d)
+    tl = torch.from_numpy(tls.astype(np.int32)).to(dev)
+    sel = list(seqs)
+    inp = Hn.Inputs(r, q[sel].cpu(), k[sel].cpu(), v[sel].cpu(), vss[sel], nvs[sel], tls[sel])
+    try:
+        for budget in budgets:
+            bd = vp.make_budget(**budget)
+            cap = max(1, vp.vp_max_kept(bd, int(nvs.max())))
+            nsel = Hkv if budget.get("granularity", 0) else 1
+            out = torch.empty((B, H, D), dtype=torch.bfloat16, device=dev)
+            kept = torch.empty((B, nsel, cap), dtype=torch.int32, device=dev)
+            count = torch.empty((B, nsel), dtype=torch.int32, device=dev)
+            mass = torch.empty((B, H), dtype=torch.float32, device=dev)
+            stats = torch.empty((B, 4), dtype=torch.float32, device=dev)
+            vp.vp_decode_step(ctx, B, q, vp.kv_contiguous(k), vp.kv_contiguous(v), span, tl, bd, out, kept,
+                              cap, count, mass, stats)
+            vp.vp_check_errors(ctx)
+            torch.cuda.synchronize()
+            gpu = dict(out=out[sel].float().cpu().numpy(), kept=kept[sel].cpu().numpy(),
+                       count=count[sel].cpu().numpy(), mass=mass[sel].cpu().numpy(), stats=stats[sel].cpu().numpy())
+            for i in range(len(sel)):
+                Hn.compare_seq(inp, gpu, i, budget, rep)
+    finally:
+        vp.vp_free(ctx)
+
+
+def test_long_reasoning_full_size_layer(vp):
+    """Long reasoning: B = 8, 4096 visual + 16384 text, lognormal key norms."""
+    rep = {}
+    _device_generated(vp, W.LONG, (0, 5, 7), [W.LONG.budget], rep)
+    assert rep.get("max_out_err", 0) < 2e-2
+
+
+@pytest.mark.parametrize("nv", [6400, 16384])
+def test_sweep_points_full_size(vp, nv):
+    """The long visual spans of the sweep at full size (B = 64, 32/8 heads):
+    the adaptive budget and 5% / 50% retention (slice and chunk gathers)."""
+    r = W.sweep_recipe(nv, W.ADAPTIVE_5PCT)
+    rep = {}
+    _device_generated(vp, r, (0, 33, 63), [W.ADAPTIVE_5PCT, W.SWEEP_BUDGETS[1], W.SWEEP_BUDGETS[3]], rep)
