@@ -254,7 +254,7 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
                                     budget->granularity);
   p.hp = ctx->lay.hp;
   p.ns = pl.ns; p.nsp_max = ctx->lay.nsp_max; p.cl = pl.cl;
-  p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
+  p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice; p.split_w = pl.split_w;
   vp::encode_kv_maps(p);
   p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st; p.hmax = ctx->hmax;
 

@@ -78,6 +78,7 @@ struct StepParams {
   int nm;             // gather CTAs that also merge a slice of the text partials (0: ns == 1)
   int nc;             // gather CTAs per (sequence, kv-head) = max(nk, nm)
   int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= 256)
+  int split_w;        // weight of one score split (bulk-tensor kernel)
 };
 
 // ---------------------------------------------------------------- host planning
@@ -91,6 +92,7 @@ constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
 // several SMs, gather chunks of 256 to 1024 kept rows.
 struct Plan {
   int ns, cl, nk, nm, nc, gslice;
+  int split_w;  // weight (tiles, text tiles counting 2) of one score split
 };
 
 inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, int max_seq, int kept_cap,
@@ -134,7 +136,12 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   // Small kept sets of few sequences: one CTA per 16 output dimensions, so
   // that the whole gather is one short wave; otherwise one CTA per chunk.
   const int gslice = kept_cap <= 256 && units * (D / 16) <= slots ? 1 : 0;
-  return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), gslice};
+  // Fixed-weight splits sized for the longest sequence: shorter ones use
+  // fewer splits, so every working score CTA carries about the same work.
+  long long w_max = 2LL * ((max_seq + 31) / 32) - max_visual / 32;
+  if (w_max < 1) w_max = 1;
+  const int split_w = (int)((w_max + ns - 1) / ns);
+  return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), gslice, split_w};
 }
 
 // Workspace layout for up to `batch` sequences (offsets in bytes, 256-aligned).

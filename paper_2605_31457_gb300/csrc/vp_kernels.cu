@@ -681,7 +681,8 @@ __device__ __forceinline__ int tma_page(const KvView& kv, const StepParams& p, i
 
 // The tiles of one split.  Tiles [v0, v1) lie wholly inside the visual span
 // (K only); every other tile carries text rows (K and V).  Split s owns
-// tiles [u0, u0 + n), cut so that every split moves about the same bytes.
+// tiles [u0, u0 + n): a fixed weight per split (from the longest sequence),
+// so that every working CTA moves about the same bytes.
 struct TileRange {
   int u0, n, v0, v1;
   __device__ __forceinline__ bool text(int t) const {
@@ -689,13 +690,13 @@ struct TileRange {
     return u < v0 || u >= v1;
   }
 };
-__device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns) {
+__device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns, int split_w) {
   const int T = sq.nv + sq.tl;
   const int NTl = (T + kTmaTile - 1) / kTmaTile;
   const int v0 = (sq.vs + kTmaTile - 1) / kTmaTile;
   const int v1 = max(v0, min(NTl, (sq.vs + sq.nv) / kTmaTile));
   const int W = 2 * NTl - (v1 - v0);  // text tiles weigh 2, visual tiles 1
-  const int per = (W + ns - 1) / ns;
+  const int per = max(split_w, (W + ns - 1) / ns);  // splits past the sequence get nothing
   auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
     if (w <= 2 * v0) return (w + 1) / 2;
     if (w <= v0 + v1) return w - v0;
@@ -733,7 +734,7 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   const int G = p.G, H = p.H;
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
   const int T = sq.nv + sq.tl;
-  const TileRange tr = tma_split(sq, s, p.ns);
+  const TileRange tr = tma_split(sq, s, p.ns, p.split_w);
   const int R = p.paged ? min(kTmaTile, p.page_size) : kTmaTile;  // rows per box
   const int nb = kTmaTile / R;                                     // boxes per tile (1..4)
   int n = tr.n;

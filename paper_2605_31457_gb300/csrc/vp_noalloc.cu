@@ -179,7 +179,7 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
                                     budget->granularity);
   p.hp = L.hp;
   p.ns = pl.ns; p.nsp_max = L.nsp_max; p.cl = pl.cl;
-  p.nk = pl.nk; p.nk_max = L.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
+  p.nk = pl.nk; p.nk_max = L.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice; p.split_w = pl.split_w;
   vp::encode_kv_maps(p);
   e = vp::launch_score(p, stream);
   if (e == cudaSuccess) e = vp::launch_select(p, stream);
