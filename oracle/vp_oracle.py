@@ -18,6 +18,8 @@ one decode step t (VisionPulse, Sec. 4.2-4.3 and Sec. 5.2):
   5. importance S_i = (1/H) sum_h A_{t,h}(q_t, v_i)                  (Eq. 2)
   6. X_v^t = Top-K_t(S)                                              (Eq. 3)
   7. attention of q_t over X_v^t plus all text tokens               (Sec. 4.2, Sec. 5.7)
+  8. for a layer after the anchor: attention over all text tokens and
+     the anchor's kept set, with no selection of its own         (Sec. 4.2, Sec. 5.1)
 
 Everything is float64 computed from the exact input values (bf16 or fp32
 inputs are widened without rounding).  There is no blocking, fusion or
@@ -247,3 +249,31 @@ def _attend(z, v, vis_start, vis, kept, G, per_head):
         out[h] = pruned_attention(z[h:h + 1], v[h // G:h // G + 1], keep)[0]
     return out
 
+
+
+def anchor_attention(q, k, v, vis_start: int, vis_len: int, text_len: int, kept, *,
+                     scale: float = 0.0) -> np.ndarray:
+    """Decode attention of a layer after the anchor layer (Sec. 4.2: the
+    importance scores are computed at l_a and pruning starts from l_a; Sec.
+    5.1 prunes at l_a = 17): the query attends to every text token and to the
+    visual tokens of the anchor's kept set X_v^t only, with no budget or
+    selection of its own.
+
+    q: [H, D]; k, v: [Hkv, >=T, D]; kept: a list holding one array of visual
+    indices (relative to the span) shared by all heads, or one per kv-head.
+    Returns out [H, D] float64.
+    """
+    q = np.asarray(q, dtype=np.float64)
+    H, D = q.shape
+    Hkv = k.shape[0]
+    G = H // Hkv
+    T = vis_len + text_len
+    if text_len < 1:
+        raise ValueError("text_len must count at least the current token")
+    if scale == 0.0:
+        scale = 1.0 / math.sqrt(D)
+    z = logits(q, np.asarray(k[:, :T], dtype=np.float64), scale)
+    vis = np.zeros(T, dtype=bool)
+    vis[vis_start:vis_start + vis_len] = True
+    kept = [np.asarray(s, dtype=np.int64) for s in kept]
+    return _attend(z, np.asarray(v[:, :T], dtype=np.float64), vis_start, vis, kept, G, per_head=len(kept) > 1)

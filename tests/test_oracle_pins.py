@@ -327,3 +327,52 @@ def test_empty_visual_span():
     np.testing.assert_array_equal(r["mass"], 0.0)
     ref = O.decode_step(q, k, v, 0, 0, tl, mode=O.DENSE)
     np.testing.assert_allclose(r["out"], ref["out"])
+
+
+# ------------------------------------------------- layers after the anchor layer
+
+def test_anchor_attention_with_every_visual_token_is_dense():
+    """A kept set holding the whole visual span gives textbook attention."""
+    q, k, v, vs, nv, tl = _rand_case(41, H=8, Hkv=2, D=16, n_v=25, text=9, vis_start=3, scale_q=2.0)
+    out = O.anchor_attention(q, k, v, vs, nv, tl, [np.arange(nv)])
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.tensor(q)[:, None], torch.tensor(k).repeat_interleave(4, 0),
+        torch.tensor(v).repeat_interleave(4, 0))[:, 0].numpy()
+    np.testing.assert_allclose(out, ref, rtol=1e-10, atol=1e-12)
+
+
+def test_anchor_attention_is_sdpa_over_text_and_kept_rows():
+    """Any kept set: SDPA over exactly the text rows and the kept visual rows
+    (pruned rows excluded, text rows before and after the span included)."""
+    q, k, v, vs, nv, tl = _rand_case(42, H=6, Hkv=3, D=8, n_v=17, text=8, vis_start=4, scale_q=2.0)
+    kept = np.array([0, 5, 6, 16])
+    out = O.anchor_attention(q, k, v, vs, nv, tl, [kept])
+    rows = np.r_[np.arange(vs), vs + kept, np.arange(vs + nv, nv + tl)]
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.tensor(q)[:, None], torch.tensor(k[:, rows]).repeat_interleave(2, 0),
+        torch.tensor(v[:, rows]).repeat_interleave(2, 0))[:, 0].numpy()
+    np.testing.assert_allclose(out, ref, rtol=1e-10, atol=1e-12)
+
+
+def test_anchor_attention_at_the_anchor_layer_reproduces_the_decode_step():
+    """Fed the anchor layer's own kept set, the layer-after-anchor attention
+    equals the decode step's output at that layer (both granularities)."""
+    q, k, v, vs, nv, tl = _rand_case(43, H=8, Hkv=2, D=16, n_v=40, text=10, vis_start=1, scale_q=3.0)
+    for gran in (0, 1):
+        r = O.decode_step(q, k, v, vs, nv, tl, mode=O.FIXED_K, fixed_k=6, granularity=gran)
+        out = O.anchor_attention(q, k, v, vs, nv, tl, r["kept"])
+        np.testing.assert_allclose(out, r["out"], rtol=1e-12, atol=1e-12)
+
+
+def test_anchor_attention_per_kv_head_sets():
+    """One kept set per kv-head: each query head attends over its own kv-head's
+    set (SDPA per group), not over another group's."""
+    q, k, v, vs, nv, tl = _rand_case(44, H=4, Hkv=2, D=8, n_v=12, text=5, scale_q=2.0)
+    sets = [np.array([1, 2]), np.array([7, 11])]
+    out = O.anchor_attention(q, k, v, vs, nv, tl, sets)
+    for g in range(2):
+        rows = np.r_[sets[g], np.arange(nv, nv + tl)]
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.tensor(q[2 * g:2 * g + 2])[:, None], torch.tensor(k[g:g + 1, rows]).expand(2, -1, -1),
+            torch.tensor(v[g:g + 1, rows]).expand(2, -1, -1))[:, 0].numpy()
+        np.testing.assert_allclose(out[2 * g:2 * g + 2], ref, rtol=1e-10, atol=1e-12)
