@@ -32,6 +32,7 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+ANCHOR_LAYER = 16  # 0-based index of the anchor layer l_a = 17 (Sec. 5.1)
 METRIC = "pruned decode-attention steps/sec and achieved HBM GB/s (% of GB300 peak) on 1 GPU"
 UNIT = "steps/s"
 NOMINAL_HBM_GBS = 8000.0
@@ -44,7 +45,7 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=None, help="timed steps (default: the workload's)")
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--workload", default="qwen7b",
-                    help="qwen7b (default) | serving | long | sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
+                    help="qwen7b (default) | qwen7b-anchor | serving | long | sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU-baseline leg")
@@ -253,7 +254,7 @@ def workload_config(r, nbuf=None):
 def pick_workload(name):
     """(recipe, default timed steps, distinct layer caches, host-generated)."""
     from paper_2605_31457_gb300 import workloads as W
-    if name == "qwen7b":
+    if name in ("qwen7b", "qwen7b-anchor"):
         return W.QWEN7B, 256, W.QWEN7B.layers, True
     if name == "serving":
         return W.SERVING, 64, 4, False
@@ -336,11 +337,28 @@ def run_ours(args, rank, world, local):
     mass = torch.empty((L, B, H), dtype=torch.float32, device=dev)
     stats = torch.empty((S, L, B, 4), dtype=torch.float32, device=dev)
 
+    # qwen7b-anchor: the anchor-layer pipeline of the paper's FastV-VP setting
+    # (Sec. 5.1, l_a = 17): layers 1-16 attend densely (the whole visual span
+    # kept), layer 17 runs the VisionPulse step, layers 18-28 reuse its kept
+    # set.  Every other workload treats each layer as its own anchor.
+    anchor = ANCHOR_LAYER if args.workload.endswith("-anchor") else None
+    if anchor is not None:
+        kept_all = torch.arange(nv_max, dtype=torch.int32, device=dev)[None, :].repeat(B, 1).contiguous()
+        count_all = vis_len.clone()
+
     def step_calls(s, stream=None):
         for layer in range(L):
-            vp.vp_decode_step(ctx, B, q_dev[s, layer], kc[layer % nbuf], vc[layer % nbuf], span, tl_steps[s], budget,
-                              out[layer], kept[layer], cap, count[s, layer], mass[layer], stats[s, layer],
-                              stream=stream)
+            kcl, vcl = kc[layer % nbuf], vc[layer % nbuf]
+            if anchor is not None and layer < anchor:
+                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], kept_all, nv_max,
+                                    count_all, out[layer], stream=stream)
+            elif anchor is not None and layer > anchor:
+                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], kept[anchor], cap,
+                                    count[s, anchor], out[layer], stream=stream)
+            else:
+                vp.vp_decode_step(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], budget,
+                                  out[layer], kept[layer], cap, count[s, layer], mass[layer], stats[s, layer],
+                                  stream=stream)
 
     # One eager step loads the kernels.  Two sets of per-step CUDA graphs: the
     # first, without timing events, gives `value` (kernels chain through
@@ -395,16 +413,22 @@ def run_ours(args, rank, world, local):
     vp.vp_check_errors(ctx)
 
     # Per-stage device times of the second pass (events recorded on the calls' stream).
-    stage = vp.vp_timing_read(ctx, S * L)[args.warmup * L:]
+    per_step = L if anchor is None else 1   # vp_decode_step calls per step (the timed ones)
+    stage = vp.vp_timing_read(ctx, S * L)[args.warmup * per_step:]
     counts = count.cpu().numpy()
-    score_bytes = gather_bytes = 0
+    score_bytes = gather_bytes = other_bytes = 0
     for s in range(args.warmup, S):
         for layer in range(L):
             for b in range(B):
-                a, c = call_bytes(r, int(nvs[b]), int(tls[b]) + s, int(counts[s, layer, b]))
-                score_bytes += a
-                gather_bytes += c
-    n_calls = args.steps * L
+                if anchor is None or layer == anchor:
+                    a, c = call_bytes(r, int(nvs[b]), int(tls[b]) + s, int(counts[s, layer, b]))
+                    score_bytes += a
+                    gather_bytes += c
+                else:  # the visual rows read: all of them before the anchor, the kept ones after
+                    nkv = int(nvs[b]) if layer < anchor else int(counts[s, anchor, b])
+                    a, c = call_bytes(r, 0, int(tls[b]) + s, 0)
+                    other_bytes += a + c + 2 * nkv * r.kv_heads * r.head_dim * 2
+    n_calls = args.steps * per_step
     score_ms = sum(x[0] for x in stage)
     select_ms = sum(x[1] for x in stage)
     gather_ms = sum(x[2] for x in stage)
@@ -413,8 +437,9 @@ def run_ours(args, rank, world, local):
     traffic = committed_traffic()
     ms_per_step = elapsed_ms / args.steps
     value = world * args.steps / (elapsed_ms * 1e-3)
-    step_gbs = (score_bytes + gather_bytes) / (elapsed_ms * 1e-3) / 1e9
-    kept_frac = float(counts[args.warmup:].sum() / (args.steps * L * nvs.sum()))
+    step_gbs = (score_bytes + gather_bytes + other_bytes) / (elapsed_ms * 1e-3) / 1e9
+    kept_layers = list(range(L)) if anchor is None else [anchor]
+    kept_frac = float(counts[args.warmup:, kept_layers].sum() / (args.steps * len(kept_layers) * nvs.sum()))
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -423,7 +448,7 @@ def run_ours(args, rank, world, local):
         "config": dict(workload_config(r, nbuf), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
         "hbm": {"achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
                 "frac_of_nominal_8tbs": step_gbs / NOMINAL_HBM_GBS,
-                "bytes_per_step": (score_bytes + gather_bytes) / args.steps,
+                "bytes_per_step": (score_bytes + gather_bytes + other_bytes) / args.steps,
                 "note": "whole step: algorithmic bytes (all visual K + kept visual V + text K/V + q + out) / step time"},
         "roofline": {"kernel": "k_score", "bound": "hbm", "achieved": achieved, "peak": peak,
                      "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
@@ -436,9 +461,16 @@ def run_ours(args, rank, world, local):
                                "gather": gather_ms * 1e3 / n_calls,
                                "timed_pass_ms_per_step": timed_ms / args.steps},
         "avg_retention": kept_frac,
-        "gpu_launches": 3 * n_calls,
+        "gpu_launches": 3 * n_calls + (0 if anchor is None else 2 * args.steps * (L - 1)),
         "clocks": clocks,
     }
+    if anchor is not None:
+        line["config"]["pipeline"] = (f"anchor layer {anchor + 1} of {L}: layers 1-{anchor} dense attention "
+                                      f"(vp_decode_gather, whole visual span kept), layer {anchor + 1} "
+                                      f"vp_decode_step, layers {anchor + 2}-{L} vp_decode_gather on its kept set")
+        line["roofline"]["timing"] += "; only the anchor layer's call is timed per kernel"
+        line["hbm"]["note"] = ("whole step: algorithmic bytes (dense layers: all K/V; anchor layer: all visual K + "
+                               "kept visual V + text K/V; later layers: kept visual K/V + text K/V; q + out) / step time")
     default = args.workload == "qwen7b"
     if not args.no_e2e and default:
         line["e2e"] = e2e_leg(args, r, vp, ctx, dev, q_dev.cpu(), ks, vs_, kc, vc, span, budget, cap, world)

@@ -149,6 +149,35 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
                          int32_t* kept_idx, int32_t kept_cap, int32_t* kept_count,
                          float* mass, float* mass_stats, void* cuda_stream);
 
+/*
+ * Decode attention of a layer after the anchor layer (Sec. 4.2: importance is
+ * computed at the anchor layer l_a and pruning starts from l_a; Sec. 5.1
+ * prunes at l_a = 17).  The query attends to every text token of the cache
+ * and to the visual tokens of a kept set produced by vp_decode_step at the
+ * anchor layer of the same decode step; no budget or selection is computed,
+ * and the visual K and V rows outside the kept set are never read.
+ *   q, k_cache, v_cache, visual_span, text_len   as for vp_decode_step (this
+ *                layer's query and caches; the same spans and lengths).
+ *   kept_idx     int32 [batch][kept_cap], or [batch][Hkv][kept_cap] when
+ *                granularity = 1: the anchor's kept visual indices (relative
+ *                to vis_start, ascending as vp_decode_step writes them).
+ *   kept_count   int32 [batch] (granularity 1: [batch][Hkv]): how many of the
+ *                slots are used; 0 <= kept_count <= min(kept_cap, vis_len).
+ *   granularity  0: one kept set per sequence; 1: one per kv-head.
+ *   scale        logit scale; 0 means 1/sqrt(D).
+ *   out          [batch][H][D] cfg.dtype.
+ * Requires bf16 caches whose layout a tensor map describes (any order of the
+ * sequence, kv-head and token axes; pages of at least 8 tokens), else
+ * VP_ERR_UNSUPPORTED.  Kept indices outside [0, vis_len) are skipped and
+ * flagged (vp_check_errors).  Uses the context's workspace: calls on one
+ * context must not overlap with each other or with vp_decode_step.
+ */
+vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
+                           const vp_kv* k_cache, const vp_kv* v_cache,
+                           const vp_span* visual_span, const int32_t* text_len,
+                           const int32_t* kept_idx, int32_t kept_cap, const int32_t* kept_count,
+                           int32_t granularity, float scale, void* out, void* cuda_stream);
+
 /* Largest K_t the budget can produce for n_visual tokens (the kept_cap a
  * caller must provide); -1 for an invalid budget.  Host only, no CUDA. */
 int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual);

@@ -1,6 +1,7 @@
 // Host side of libvp: argument checking, workspace ownership, launch planning
 // and the extern "C" entry points declared in include/vp.h.
 #include <cuda_runtime.h>
+#include <cmath>
 #include <math.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -284,6 +285,83 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
 
 const char* vp_last_error(const vp_ctx* ctx) {
   return ctx ? ctx->last_error.c_str() : g_init_error.c_str();
+}
+
+vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
+                           const vp_kv* k_cache, const vp_kv* v_cache,
+                           const vp_span* visual_span, const int32_t* text_len,
+                           const int32_t* kept_idx, int32_t kept_cap, const int32_t* kept_count,
+                           int32_t granularity, float scale, void* out, void* cuda_stream) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  ctx->last_error.clear();
+  const vp_config& c = ctx->cfg;
+  if (batch < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: batch < 0");
+  if (batch > c.max_batch) return fail(ctx, VP_ERR_CAPACITY, "vp_decode_gather: batch exceeds max_batch");
+  if (granularity != 0 && granularity != 1) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: granularity must be 0 or 1");
+  if (kept_cap < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: kept_cap < 0");
+  if (!(scale >= 0.f) || !std::isfinite(scale)) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: scale must be finite and >= 0");
+  if (c.dtype != VP_BF16) return fail(ctx, VP_ERR_UNSUPPORTED, "vp_decode_gather: needs bf16 caches");
+  if (batch == 0) return VP_OK;
+  if (!q || !out || !text_len || !visual_span || !visual_span->vis_start || !visual_span->vis_len || !kept_count ||
+      (kept_cap > 0 && !kept_idx))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: NULL tensor argument");
+  if (!aligned16(q) || !aligned16(out)) return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: q and out must be 16-byte aligned");
+  std::string why;
+  if (!kv_ok(ctx, k_cache, "k_cache", &why) || !kv_ok(ctx, v_cache, "v_cache", &why))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_decode_gather: " + why);
+
+  const int H = c.num_q_heads, Hkv = c.num_kv_heads, D = c.head_dim;
+  vp::StepParams p;
+  memset(&p, 0, sizeof p);
+  p.dtype = c.dtype;
+  p.B = batch; p.H = H; p.Hkv = Hkv; p.G = H / Hkv; p.D = D;
+  p.max_visual = c.max_visual; p.max_seq = c.max_seq;
+  p.paged = c.paged; p.page_size = c.paged ? c.page_size : 1;
+  while ((1 << p.page_shift) < p.page_size) ++p.page_shift;
+  p.q = q;
+  p.k = vp::KvView{k_cache->data, k_cache->stride_b, k_cache->stride_h, k_cache->stride_t,
+                   k_cache->block_table, k_cache->max_pages, k_cache->num_pages};
+  p.v = vp::KvView{v_cache->data, v_cache->stride_b, v_cache->stride_h, v_cache->stride_t,
+                   v_cache->block_table, v_cache->max_pages, v_cache->num_pages};
+  p.vis_start = visual_span->vis_start;
+  p.vis_len = visual_span->vis_len;
+  p.text_len = text_len;
+  p.anchor = 1;
+  p.granularity = granularity;
+  p.inv_tau = 1.f;
+  p.c_log2 = (scale > 0.f ? scale : 1.0f / sqrtf((float)D)) * 1.4426950408889634f;
+  p.kept_idx = const_cast<int32_t*>(kept_idx);
+  p.kept_cap = kept_cap;
+  p.kept_count = const_cast<int32_t*>(kept_count);
+  p.out = out;
+  p.z_ws = ctx->z_ws; p.split_st = ctx->split_st; p.split_o = ctx->split_o;
+  p.gpart_o = ctx->gpart_o; p.gpart_st = ctx->gpart_st; p.tickets = ctx->tickets; p.err = ctx->err;
+  p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st; p.hmax = ctx->hmax;
+  // Score splits as planned for the decode step; their weight covers the
+  // cache outside the visual span plus the kept rows.  The merge of the
+  // splits is the chunk gather with no kept chunks.
+  const vp::Plan pl = vp::make_plan(batch, Hkv, D, ctx->num_sms, c.max_visual, c.max_seq, 0, granularity);
+  p.hp = ctx->lay.hp;
+  p.ns = pl.ns; p.nsp_max = ctx->lay.nsp_max; p.cl = 1;
+  {
+    long long w = 2LL * ((c.max_seq + 31) / 32 - c.max_visual / 32 + (kept_cap + 31) / 32);
+    if (w < 1) w = 1;
+    p.split_w = (int)((w + pl.ns - 1) / pl.ns);
+  }
+  p.nk = 0; p.nk_max = ctx->lay.nk_max;
+  p.nm = pl.ns > 1 ? (D / 16 < 8 ? D / 16 : 8) : 0;
+  p.nc = p.nm > 0 ? p.nm : 1;
+  p.gslice = 0;
+  vp::encode_kv_maps(p);
+  if (!p.use_tma)
+    return fail(ctx, VP_ERR_UNSUPPORTED, "vp_decode_gather: the cache layout needs the bulk-tensor path "
+                "(token axis not outermost, pages of at least 8 tokens)");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = vp::launch_score(p, st);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: score kernel launch", e);
+  e = vp::launch_gather(p, st);
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: merge kernel launch", e);
+  return VP_OK;
 }
 
 vp_status vp_check_errors(vp_ctx* ctx, void* cuda_stream) {

@@ -36,6 +36,7 @@ struct StepParams {
   CUtensorMap tmk;  // 64-byte aligned type
   CUtensorMap tmv;
   int use_tma;
+  int anchor;  // 1: a layer after the anchor layer -- text plus the given kept set, no selection
   int tpos, gpos, bpos;  // descriptor dimension (1..3) of the token, kv-head and sequence/page axes
   // shapes
   int dtype;  // 0 = bf16, 1 = fp32 (vp_dtype)

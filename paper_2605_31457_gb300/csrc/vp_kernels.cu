@@ -211,6 +211,12 @@ __device__ __forceinline__ void cp_async4(unsigned dst, const void* src) {
 __device__ __forceinline__ void cp_async_arrive(uint64_t* bar) {
   asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(smem_u32(bar)) : "memory");
 }
+// The same arrive-on, but the barrier's pending count is raised first, so
+// the arrival needs no room in the barrier's count (a normal arrival still
+// completes the phase once the copies have landed).
+__device__ __forceinline__ void cp_async_arrive_counted(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
 
 struct Seq {
   int vs, nv, tl;
@@ -681,20 +687,41 @@ __device__ __forceinline__ int tma_page(const KvView& kv, const StepParams& p, i
 
 // The tiles of one split.  Tiles [v0, v1) lie wholly inside the visual span
 // (K only); every other tile carries text rows (K and V).  Split s owns
-// tiles [u0, u0 + n): a fixed weight per split (from the longest sequence),
-// so that every working CTA moves about the same bytes.
+// list entries [u0, u0 + n): a fixed weight per split (from the longest
+// sequence), so that every working CTA moves about the same bytes.  For a
+// layer after the anchor layer (ntext >= 0) the list is the cache tiles
+// outside [v0, v1), then the kept visual tokens in tiles of 32, all
+// attended with K and V.
 struct TileRange {
-  int u0, n, v0, v1;
+  int u0, n, v0, v1, ntext;
   __device__ __forceinline__ bool text(int t) const {
     const int u = u0 + t;
-    return u < v0 || u >= v1;
+    return ntext >= 0 || u < v0 || u >= v1;
+  }
+  __device__ __forceinline__ bool kept(int t) const { return ntext >= 0 && u0 + t >= ntext; }
+  // Cache tile of entry t (not for kept entries).
+  __device__ __forceinline__ int tile(int t) const {
+    const int u = u0 + t;
+    return (ntext >= 0 && u >= v0) ? u + (v1 - v0) : u;
   }
 };
-__device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns, int split_w) {
+__device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns, int split_w, int n_kept) {
   const int T = sq.nv + sq.tl;
   const int NTl = (T + kTmaTile - 1) / kTmaTile;
   const int v0 = (sq.vs + kTmaTile - 1) / kTmaTile;
   const int v1 = max(v0, min(NTl, (sq.vs + sq.nv) / kTmaTile));
+  TileRange r;
+  r.v0 = v0;
+  r.v1 = v1;
+  if (n_kept >= 0) {  // after the anchor: every entry weighs 2
+    r.ntext = NTl - (v1 - v0);
+    const int L = r.ntext + (n_kept + kTmaTile - 1) / kTmaTile;
+    const int per = max(split_w, (2 * L + ns - 1) / ns);
+    r.u0 = (min(2 * L, s * per) + 1) / 2;
+    r.n = (min(2 * L, (s + 1) * per) + 1) / 2 - r.u0;
+    return r;
+  }
+  r.ntext = -1;
   const int W = 2 * NTl - (v1 - v0);  // text tiles weigh 2, visual tiles 1
   const int per = max(split_w, (W + ns - 1) / ns);  // splits past the sequence get nothing
   auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
@@ -702,15 +729,13 @@ __device__ __forceinline__ TileRange tma_split(const Seq& sq, int s, int ns, int
     if (w <= v0 + v1) return w - v0;
     return (w + (v1 - v0) + 1) / 2;
   };
-  TileRange r;
   r.u0 = tile_of(min(W, s * per));
   r.n = tile_of(min(W, (s + 1) * per)) - r.u0;
-  r.v0 = v0;
-  r.v1 = v1;
   return r;
 }
 
-template <int D, int NT, int NW, int S>
+// ANCHOR: a layer after the anchor layer (text plus the given kept set).
+template <int D, int NT, int NW, int S, bool ANCHOR>
 __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant__ StepParams p) {
   using C = TmaCfg<D, NT, NW, S>;
   constexpr int GM = C::GM;
@@ -734,20 +759,36 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   const int G = p.G, H = p.H;
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
   const int T = sq.nv + sq.tl;
-  const TileRange tr = tma_split(sq, s, p.ns, p.split_w);
+  unsigned err = 0;
+  // After the anchor layer: the kept set of this sequence (or kv-head).
+  int n_kept = -1;
+  const int32_t* kept_rows = nullptr;
+  if (ANCHOR) {
+    const int sel = p.granularity ? b * p.Hkv + g : b;
+    const int c = __ldg(p.kept_count + sel);
+    if (c < 0 || c > min(p.kept_cap, sq.nv)) err |= ERR_KEPT;
+    n_kept = max(0, min(c, min(p.kept_cap, sq.nv)));
+    kept_rows = p.kept_idx + (int64_t)sel * p.kept_cap;
+  }
+  const TileRange tr = tma_split(sq, s, p.ns, p.split_w, n_kept);
+  // Entry kinds, constant-folded for the decode step.
+  auto is_text = [&](int t) { return ANCHOR || tr.text(t); };
+  auto is_kept = [&](int t) { return ANCHOR && tr.kept(t); };
+  auto tile_at = [&](int t) { return ANCHOR ? tr.tile(t) : tr.u0 + t; };
   const int R = p.paged ? min(kTmaTile, p.page_size) : kTmaTile;  // rows per box
   const int nb = kTmaTile / R;                                     // boxes per tile (1..4)
   int n = tr.n;
-  unsigned err = 0;
   if (p.paged) {
     if (n * nb > kTmaMaxBoxes) {  // the host plan keeps every CTA below this
       err |= ERR_PAGE;
       n = 0;
     }
     for (int i = tid; i < n * nb; i += C::THREADS) {
-      const int t = i / nb, pos = (tr.u0 + t) * kTmaTile + (i % nb) * R;
+      const int t = i / nb;
+      if (is_kept(t)) continue;  // kept rows find their pages when issued
+      const int pos = tile_at(t) * kTmaTile + (i % nb) * R;
       kpg[i] = pos < T ? tma_page(p.k, p, b, pos) : -2;
-      vpg[i] = (pos < T && tr.text(t)) ? tma_page(p.v, p, b, pos) : 0;
+      vpg[i] = (pos < T && is_text(t)) ? tma_page(p.v, p, b, pos) : 0;
     }
   }
   __syncthreads();
@@ -759,14 +800,52 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   auto issue = [&]() {
     while (ji < nj) {
       const int t = warp + NW * ji;
-      const bool text = tr.text(t);
+      const bool text = is_text(t);
       const int need = text ? 2 : 1;
       if (qi + need - qf > S) break;
       // The slots were last read by this warp's ldmatrix (generic proxy).
       fence_proxy_async();
       __syncwarp();
-      if (lane == 0) {
-        const int p0 = (tr.u0 + t) * kTmaTile;
+      if (is_kept(t)) {
+        // Kept visual rows (after the anchor layer): each lane finds one row;
+        // the warp copies K and V in 16-byte pieces, two rows per instruction,
+        // into the swizzled layout of the tensor copies.
+        const int r = (tr.u0 + t - tr.ntext) * kTmaTile + lane;
+        int i = r < n_kept ? __ldg(kept_rows + r) : -1;
+        if (r < n_kept && (i < 0 || i >= sq.nv)) { err |= ERR_KEPT; i = -1; }
+        const __nv_bfloat16* kr = nullptr;
+        const __nv_bfloat16* vr = nullptr;
+        if (i >= 0) {
+          kr = kv_row<__nv_bfloat16>(p.k, p, b, g, sq.vs + i);
+          vr = kv_row<__nv_bfloat16>(p.v, p, b, g, sq.vs + i);
+          if (!kr || !vr) { err |= ERR_PAGE; kr = vr = nullptr; }
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, kr != nullptr);
+        const int ks = qi % S, vs = (qi + 1) % S;
+        constexpr int PPR = 2 * D / 16, RPI = 32 / PPR;
+        const unsigned kt = smem_u32(ring + ks * C::SLOT), vt = smem_u32(ring + vs * C::SLOT);
+        const unsigned long long ka = reinterpret_cast<unsigned long long>(kr);
+        const unsigned long long va = reinterpret_cast<unsigned long long>(vr);
+#pragma unroll
+        for (int jj = 0; jj < 32 / RPI; ++jj) {
+          const int row = jj * RPI + lane / PPR;
+          const unsigned off = swz_off<C::HALF_BYTES>(row, 8 * (lane % PPR));
+          const unsigned long long a1 = __shfl_sync(0xffffffffu, ka, row);
+          const unsigned long long a2 = __shfl_sync(0xffffffffu, va, row);
+          if (a1) cp_async16(kt + off, reinterpret_cast<const char*>(a1) + (lane % PPR) * 16);
+          if (a2) cp_async16(vt + off, reinterpret_cast<const char*>(a2) + (lane % PPR) * 16);
+        }
+        cp_async_arrive_counted(full + ks);
+        cp_async_arrive_counted(full + vs);
+        __syncwarp();
+        if (lane == 0) {
+          rowmask[ks] = m;
+          mbar_expect_tx(full + ks, 0u);
+          mbar_expect_tx(full + vs, 0u);
+        }
+      } else if (lane == 0) {
+        const int p0 = tile_at(t) * kTmaTile;
+
         const int nvalid = min(kTmaTile, T - p0);
         uint32_t mask = nvalid >= 32 ? 0xffffffffu : ((1u << nvalid) - 1u);
         const int ks = qi % S, vs = (qi + 1) % S;
@@ -851,11 +930,12 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
 
   for (int j = 0; j < nj; ++j) {
     const int t = warp + NW * j;
-    const bool text = tr.text(t);
+    const bool text = is_text(t);
     const int ks_ = qc % S;
     if (!mbar_wait(full + ks_, (qc / S) & 1)) { timed_out = true; break; }
     const uint32_t mask = rowmask[ks_];
-    const int p0 = (tr.u0 + t) * kTmaTile;
+    const bool kept_tile = is_kept(t);
+    const int p0 = kept_tile ? 0 : tile_at(t) * kTmaTile;
     const unsigned kt = smem_u32(ring + ks_ * C::SLOT);
 
     // ---- QK for both 16-row halves of the tile, then refill the K slot
@@ -887,14 +967,18 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
         const int row = 16 * sb + gr + 8 * (e >> 1);
         const int pos = p0 + row;
         const bool valid = (mask >> row) & 1u;
-        const bool vis = valid && (unsigned)(pos - sq.vs) < (unsigned)sq.nv;
+        // A cache row inside the visual span is visual; after the anchor
+        // layer it is left out (its kept tokens come as kept rows).
+        const bool inspan = !kept_tile && (unsigned)(pos - sq.vs) < (unsigned)sq.nv;
+        const bool vis = !ANCHOR && valid && inspan;
+        const bool txt = valid && !inspan;
         any_vis |= vis;
 #pragma unroll
         for (int nn = 0; nn < NT; ++nn) {
           const bool hv = (8 * nn + 2 * tg + (e & 1)) < G;
           const float z = c[sb][nn][e] * p.c_log2;
           zv[sb][nn][e] = (vis && hv) ? z : -CUDART_INF_F;
-          zt[sb][nn][e] = (valid && !vis && hv) ? z : -CUDART_INF_F;
+          zt[sb][nn][e] = (txt && hv) ? z : -CUDART_INF_F;
         }
         if (vis) {
           float* zrow = p.z_ws + ((int64_t)b * p.max_visual + (pos - sq.vs)) * p.hp + g * G;
@@ -1846,13 +1930,19 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   float (*tl)[kNsMax] = tw + GM;
   // (b) first: it reads only the score kernel's partials, complete before the
   // select kernel lets this grid start.  Its shared memory is the ring's.
-  if (c < p.nm) {
+  // After the anchor layer no select kernel runs in between: there (b)
+  // waits for the score kernel like everything else.
+  if (c < p.nm && !p.anchor) {
     gather_text_slice<D, GM, C::THREADS>(p, c, hrow0, tw, tl);
     fence_proxy_async();
     __syncthreads();
   }
   pdl_wait();
   pdl_trigger();
+  if (c < p.nm && p.anchor) {
+    gather_text_slice<D, GM, C::THREADS>(p, c, hrow0, tw, tl);
+    __syncthreads();
+  }
   const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
   unsigned err = 0;
   bool timed_out = false;
@@ -2280,8 +2370,12 @@ cudaError_t launch_score_d(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.ns, p.Hkv, p.B);
   if (p.dtype == 0 && p.use_tma) {
     constexpr int NW = kTmaWarps, S = tma_slots<D>();
-    if (p.G <= 8) return launch_ex(k_score_tma<D, 1, NW, S>, grid, dim3(32 * NW), tma_smem<D, 1>(), st, 1, p);
-    return launch_ex(k_score_tma<D, 2, NW, S>, grid, dim3(32 * NW), tma_smem<D, 2>(), st, 1, p);
+    if (p.anchor) {
+      if (p.G <= 8) return launch_ex(k_score_tma<D, 1, NW, S, true>, grid, dim3(32 * NW), tma_smem<D, 1>(), st, 1, p);
+      return launch_ex(k_score_tma<D, 2, NW, S, true>, grid, dim3(32 * NW), tma_smem<D, 2>(), st, 1, p);
+    }
+    if (p.G <= 8) return launch_ex(k_score_tma<D, 1, NW, S, false>, grid, dim3(32 * NW), tma_smem<D, 1>(), st, 1, p);
+    return launch_ex(k_score_tma<D, 2, NW, S, false>, grid, dim3(32 * NW), tma_smem<D, 2>(), st, 1, p);
   }
   if (p.dtype == 0) {
     if (p.G <= 8) return launch_ex(k_score_mma<D, 1>, grid, dim3(kThreads), mma_smem<D, 1>(), st, 1, p);
@@ -2325,10 +2419,14 @@ cudaError_t configure_fixed_kernels() {
   VP_SET((k_gather_mma<128, 2>), (GmCfg<128, 2>::SMEM));
   VP_SET((k_gather_mma<64, 1>), (GmCfg<64, 1>::SMEM));
   VP_SET((k_gather_mma<64, 2>), (GmCfg<64, 2>::SMEM));
-  VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 1>()));
-  VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>()>), (tma_smem<128, 2>()));
-  VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>()>), (tma_smem<64, 1>()));
-  VP_SET((k_score_tma<64, 2, kTmaWarps, tma_slots<64>()>), (tma_smem<64, 2>()));
+  VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>(), false>), (tma_smem<128, 1>()));
+  VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>(), false>), (tma_smem<128, 2>()));
+  VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>(), false>), (tma_smem<64, 1>()));
+  VP_SET((k_score_tma<64, 2, kTmaWarps, tma_slots<64>(), false>), (tma_smem<64, 2>()));
+  VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>(), true>), (tma_smem<128, 1>()));
+  VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>(), true>), (tma_smem<128, 2>()));
+  VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>(), true>), (tma_smem<64, 1>()));
+  VP_SET((k_score_tma<64, 2, kTmaWarps, tma_slots<64>(), true>), (tma_smem<64, 2>()));
   VP_SET((k_score_mma<128, 1>), (mma_smem<128, 1>()));
   VP_SET((k_score_mma<128, 2>), (mma_smem<128, 2>()));
   VP_SET((k_score_mma<64, 1>), (mma_smem<64, 1>()));

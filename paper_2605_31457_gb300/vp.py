@@ -70,6 +70,10 @@ lib.vp_decode_step.argtypes = [_P, ctypes.c_int32, _P, ctypes.POINTER(vp_kv), ct
                                ctypes.POINTER(vp_span), _P, ctypes.POINTER(vp_budget), _P,
                                _P, ctypes.c_int32, _P, _P, _P, _P]
 lib.vp_decode_step.restype = ctypes.c_int
+lib.vp_decode_gather.argtypes = [_P, ctypes.c_int32, _P, ctypes.POINTER(vp_kv), ctypes.POINTER(vp_kv),
+                                 ctypes.POINTER(vp_span), _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
+                                 ctypes.c_float, _P, _P]
+lib.vp_decode_gather.restype = ctypes.c_int
 lib.vp_max_kept.argtypes = [ctypes.POINTER(vp_budget), ctypes.c_int32]
 lib.vp_max_kept.restype = ctypes.c_int32
 lib.vp_last_error.argtypes = [_P]
@@ -127,6 +131,22 @@ def vp_decode_step(ctx, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span: v
                             ctypes.byref(visual_span), _ptr(text_len), ctypes.byref(budget), _ptr(out),
                             _ptr(kept_idx), int(kept_cap), _ptr(kept_count), _ptr(mass),
                             _ptr(mass_stats), ctypes.c_void_p(stream))
+    return _check(st, ctx) if check else st
+
+
+def vp_decode_gather(ctx, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span: vp_span, text_len,
+                     kept_idx, kept_cap, kept_count, out, granularity=0, scale=0.0, stream=None, check=True):
+    """Enqueues the attention of a layer after the anchor layer over every text
+    token and the anchor's kept set (kept_idx / kept_count as vp_decode_step
+    wrote them).  Tensors are torch CUDA tensors."""
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream().cuda_stream
+    elif hasattr(stream, "cuda_stream"):
+        stream = stream.cuda_stream
+    st = lib.vp_decode_gather(ctx, int(batch), _ptr(q), ctypes.byref(k_cache), ctypes.byref(v_cache),
+                              ctypes.byref(visual_span), _ptr(text_len), _ptr(kept_idx), int(kept_cap),
+                              _ptr(kept_count), int(granularity), float(scale), _ptr(out), ctypes.c_void_p(stream))
     return _check(st, ctx) if check else st
 
 

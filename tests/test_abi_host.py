@@ -23,7 +23,7 @@ def _declared():
 
 def test_header_declares_the_boundary():
     assert {"vp_init", "vp_decode_step", "vp_free", "vp_last_error", "vp_check_errors",
-            "vp_max_kept"} <= _declared()
+            "vp_max_kept", "vp_decode_gather"} <= _declared()
 
 
 def test_library_exports_every_declared_symbol(lib):
@@ -58,6 +58,8 @@ def test_null_context_and_null_free(lib):
                                 None, 0, None, None, None, None)
     assert st == lib.VP_ERR_NOT_INITIALIZED
     assert lib.lib.vp_check_errors(None, None) == lib.VP_ERR_NOT_INITIALIZED
+    st = lib.lib.vp_decode_gather(None, 1, None, None, None, None, None, None, 0, None, 0, 0.0, None, None)
+    assert st == lib.VP_ERR_NOT_INITIALIZED
     lib.vp_free(None)
 
 
