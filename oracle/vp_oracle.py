@@ -20,6 +20,8 @@ one decode step t (VisionPulse, Sec. 4.2-4.3 and Sec. 5.2):
   7. attention of q_t over X_v^t plus all text tokens               (Sec. 4.2, Sec. 5.7)
   8. for a layer after the anchor: attention over all text tokens and
      the anchor's kept set, with no selection of its own         (Sec. 4.2, Sec. 5.1)
+  9. the active visual token count N_act(delta) and the per-token
+     activity flags behind persistent inactivity                   (Sec. 4.3, App. B)
 
 Everything is float64 computed from the exact input values (bf16 or fp32
 inputs are widened without rounding).  There is no blocking, fusion or
@@ -277,3 +279,18 @@ def anchor_attention(q, k, v, vis_start: int, vis_len: int, text_len: int, kept,
     vis[vis_start:vis_start + vis_len] = True
     kept = [np.asarray(s, dtype=np.int64) for s in kept]
     return _attend(z, np.asarray(v[:, :T], dtype=np.float64), vis_start, vis, kept, G, per_head=len(kept) > 1)
+
+
+def active_count(s: np.ndarray, delta: float):
+    """Active visual token count of Sec. 4.3 (the equation defining
+    N_act^t(delta)): how many visual tokens have a head-averaged attention
+    probability (the S of Eq. 2) above delta, and which ones.  Scores and the
+    threshold are compared in float32, the precision the kernel decides in.
+    A token whose flag stays False at every step of a decode is persistently
+    inactive (App. B, "Persistent visual redundancy during reasoning").
+
+    s: [N_v] importance scores (or [Hkv, N_v] for per-kv-head selection).
+    Returns (N_act, boolean activity flags of the same shape as s).
+    """
+    active = np.asarray(s, dtype=np.float32) > np.float32(delta)
+    return active.sum(axis=-1), active

@@ -376,3 +376,41 @@ def test_anchor_attention_per_kv_head_sets():
             torch.tensor(q[2 * g:2 * g + 2])[:, None], torch.tensor(k[g:g + 1, rows]).expand(2, -1, -1),
             torch.tensor(v[g:g + 1, rows]).expand(2, -1, -1))[:, 0].numpy()
         np.testing.assert_allclose(out[2 * g:2 * g + 2], ref, rtol=1e-10, atol=1e-12)
+
+
+# ------------------------------------------------------- active visual tokens
+
+def test_active_count_zero_query_closed_form():
+    """q = 0: every score is 1/T, so every visual token is active exactly when
+    1/T exceeds delta."""
+    q, k, v, vs, nv, tl = _rand_case(51, n_v=20, text=6)
+    r = O.decode_step(np.zeros_like(q), k, v, vs, nv, tl)
+    T = nv + tl
+    n, act = O.active_count(r["s"], 0.9 / T)
+    assert n == nv and act.all()
+    n, act = O.active_count(r["s"], 1.1 / T)
+    assert n == 0 and not act.any()
+
+
+def test_active_count_brute_force_and_limits():
+    """Count by hand on a random case; delta below every score counts all
+    tokens, delta at the largest score counts none; monotone in delta."""
+    q, k, v, vs, nv, tl = _rand_case(52, n_v=30, text=5, scale_q=3.0)
+    s = O.decode_step(q, k, v, vs, nv, tl)["s"]
+    for delta in (1e-4, 1e-3, 1e-2, 5e-2):
+        n, act = O.active_count(s, delta)
+        assert n == sum(1 for x in s if np.float32(x) > np.float32(delta))
+        assert list(np.flatnonzero(act)) == [i for i in range(nv) if np.float32(s[i]) > np.float32(delta)]
+    assert O.active_count(s, 0.0)[0] == nv
+    assert O.active_count(s, float(np.float32(s.max())))[0] == 0
+    counts = [O.active_count(s, d)[0] for d in np.geomspace(1e-6, 1.0, 25)]
+    assert all(a >= b for a, b in zip(counts, counts[1:]))
+
+
+def test_active_count_per_kv_head():
+    q, k, v, vs, nv, tl = _rand_case(53, H=4, Hkv=2, n_v=16, text=4, scale_q=2.0)
+    s = O.decode_step(q, k, v, vs, nv, tl, granularity=1)["s"]
+    n, act = O.active_count(s, 0.02)
+    assert n.shape == (2,) and act.shape == (2, nv)
+    for g in range(2):
+        assert n[g] == (s[g].astype(np.float32) > np.float32(0.02)).sum()
