@@ -178,6 +178,25 @@ vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
                            const int32_t* kept_idx, int32_t kept_cap, const int32_t* kept_count,
                            int32_t granularity, float scale, void* out, void* cuda_stream);
 
+/*
+ * Diagnostics of the step-wise analysis (Sec. 4.3, App. B); off by default.
+ * Once set on a context, every later vp_decode_step on it also
+ *   - writes n_act (int32 [batch]; granularity 1: [batch][Hkv]) = N_act(delta),
+ *     the number of visual tokens whose head-averaged attention probability
+ *     (the S_i of Eq. 2, compared in float32) exceeds delta;
+ *   - sets, in active_bits (uint32 [batch][words]; granularity 1:
+ *     [batch][Hkv][words]; words = (max_visual + 31) / 32), bit i % 32 of
+ *     word i / 32 for every visual token i with S_i > delta.  Bits are only
+ *     ever set: zero the array when a sequence starts; a token whose bit is
+ *     still 0 when its decode ends was never active (persistently inactive,
+ *     App. B).
+ * Either pointer may be NULL; both NULL turns the diagnostics off.  delta
+ * must be finite and > 0 (else VP_ERR_INVALID_ARG).  The arrays are
+ * caller-owned device memory, 4-byte aligned, valid while set; the setting is
+ * read when a call is enqueued (a captured graph keeps the pointers it saw).
+ */
+vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t* active_bits);
+
 /* Largest K_t the budget can produce for n_visual tokens (the kept_cap a
  * caller must provide); -1 for an invalid budget.  Host only, no CUDA. */
 int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual);

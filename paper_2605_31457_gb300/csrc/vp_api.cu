@@ -29,6 +29,9 @@ struct vp_ctx {
   float* mt_o = nullptr;
   float* mt_st = nullptr;
   float* hmax = nullptr;
+  float diag_delta = 0.f;          // diagnostics (vp_set_diagnostics)
+  int32_t* diag_n_act = nullptr;
+  uint32_t* diag_bits = nullptr;
   unsigned* tickets = nullptr;
   unsigned* err = nullptr;
   std::string last_error;
@@ -258,6 +261,12 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice; p.split_w = pl.split_w;
   vp::encode_kv_maps(p);
   p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st; p.hmax = ctx->hmax;
+  if (ctx->diag_n_act || ctx->diag_bits) {
+    memcpy(&p.act_delta_bits, &ctx->diag_delta, sizeof(float));
+    p.n_act = ctx->diag_n_act;
+    p.act_bits = ctx->diag_bits;
+    p.act_words = (c.max_visual + 31) / 32;
+  }
 
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   cudaEvent_t* tev = nullptr;
@@ -361,6 +370,19 @@ vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: score kernel launch", e);
   e = vp::launch_gather(p, st);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: merge kernel launch", e);
+  return VP_OK;
+}
+
+vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t* active_bits) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  ctx->last_error.clear();
+  if ((n_act || active_bits) && !(delta > 0.f && std::isfinite(delta)))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_set_diagnostics: delta must be finite and > 0");
+  if ((n_act && (reinterpret_cast<uintptr_t>(n_act) & 3u)) || (active_bits && (reinterpret_cast<uintptr_t>(active_bits) & 3u)))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_set_diagnostics: arrays must be 4-byte aligned");
+  ctx->diag_delta = delta;
+  ctx->diag_n_act = n_act;
+  ctx->diag_bits = active_bits;
   return VP_OK;
 }
 

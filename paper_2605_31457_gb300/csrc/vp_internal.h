@@ -70,6 +70,11 @@ struct StepParams {
   float* mt_o;        // [max_batch][H][D] text output merged over the splits
   float* mt_st;       // [max_batch][H][2] its {max, sum}
   float* hmax;        // [max_batch][H] largest logit of every head over all tokens (log2 units)
+  // Diagnostics (Sec. 4.3, App. B), off when both pointers are NULL.
+  unsigned act_delta_bits;  // float bits of delta (> 0): a score S_i is active when its bits are larger
+  int32_t* n_act;           // [B][nsel] N_act(delta)
+  uint32_t* act_bits;       // [B][nsel][act_words] activity bits, OR-accumulated
+  int act_words;
   unsigned* tickets;  // [max_batch][Hkv] (zero between calls)
   unsigned* err;      // device error word
   int hp;             // z_ws row stride (H rounded up to a multiple of 4)

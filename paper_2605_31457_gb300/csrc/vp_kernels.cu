@@ -1341,11 +1341,13 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   __shared__ unsigned hist_s[3][256];  // one per radix pass, used in turn
   __shared__ int wsum_s[32];
   __shared__ int sh_i[4];
+  __shared__ int act_s, act_rank_s[8];  // active-token counts (diagnostics)
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
   const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int i = tid; i < 3 * 256; i += NTH) (&hist_s[0][0])[i] = 0;
+  if (tid == 0) act_s = 0;
   pdl_wait();
   pdl_trigger();
   const int H = p.H, ns = p.ns;
@@ -1460,6 +1462,8 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   const float inv_cnt = 1.f / (float)hcnt;
   uint32_t* key0 = ncl > 1 ? cluster.map_shared_rank(key_s, 0) : key_s;
   unsigned bad = 0;
+  const bool diag = p.n_act || p.act_bits;
+  int n_on = 0;
   for (int i = i0 + tid; i < i1; i += NTH) {
     const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
     float a = 0.f;
@@ -1490,12 +1494,27 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     const float sc = a * inv_cnt;
     if (!isfinite(sc)) bad = 1;
     key0[i] = __float_as_uint(sc);
+    if (diag && __float_as_uint(sc) > p.act_delta_bits) {  // S_i > delta (Sec. 4.3)
+      ++n_on;
+      if (p.act_bits) atomicOr(p.act_bits + ((int64_t)b * nsel + gsel) * p.act_words + (i >> 5), 1u << (i & 31));
+    }
   }
   if (bad) atomicOr(p.err, ERR_NONFINITE);
+  if (p.n_act) {  // this rank's count, into rank 0's slot
+    n_on = __reduce_add_sync(0xffffffffu, n_on);
+    if (lane == 0 && n_on) atomicAdd(&act_s, n_on);
+    __syncthreads();
+    if (tid == 0) (ncl > 1 ? cluster.map_shared_rank(act_rank_s, 0) : act_rank_s)[rank] = act_s;
+  }
   if (ncl > 1) cluster.sync();  // rank 0 now sees every key (and its own K)
   else __syncthreads();
   if (rank != 0) return;
 
+  if (p.n_act && tid == 0) {
+    int n = 0;
+    for (int r = 0; r < ncl; ++r) n += act_rank_s[r];
+    p.n_act[(int64_t)b * nsel + gsel] = n;
+  }
   const int K = sh_i[0];
   int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
 

@@ -74,6 +74,8 @@ lib.vp_decode_gather.argtypes = [_P, ctypes.c_int32, _P, ctypes.POINTER(vp_kv), 
                                  ctypes.POINTER(vp_span), _P, _P, ctypes.c_int32, _P, ctypes.c_int32,
                                  ctypes.c_float, _P, _P]
 lib.vp_decode_gather.restype = ctypes.c_int
+lib.vp_set_diagnostics.argtypes = [_P, ctypes.c_float, _P, _P]
+lib.vp_set_diagnostics.restype = ctypes.c_int
 lib.vp_max_kept.argtypes = [ctypes.POINTER(vp_budget), ctypes.c_int32]
 lib.vp_max_kept.restype = ctypes.c_int32
 lib.vp_last_error.argtypes = [_P]
@@ -148,6 +150,12 @@ def vp_decode_gather(ctx, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span:
                               ctypes.byref(visual_span), _ptr(text_len), _ptr(kept_idx), int(kept_cap),
                               _ptr(kept_count), int(granularity), float(scale), _ptr(out), ctypes.c_void_p(stream))
     return _check(st, ctx) if check else st
+
+
+def vp_set_diagnostics(ctx, delta, n_act=None, active_bits=None):
+    """Turns on (or off, with both arrays None) the N_act(delta) count and the
+    OR-accumulated activity bits of later vp_decode_step calls."""
+    return _check(lib.vp_set_diagnostics(ctx, float(delta), _ptr(n_act), _ptr(active_bits)), ctx)
 
 
 def vp_max_kept(budget: vp_budget, n_visual: int) -> int:
