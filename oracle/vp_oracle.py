@@ -56,6 +56,7 @@ ADAPTIVE = 0      # Eq. 7 with the clamp of Sec. 5.2
 FIXED_RATIO = 1   # "FastV-VP (Fix Ratio)", Sec. 5.4 / Table 2
 FIXED_K = 2       # constant Top-k budget, App. A.2
 DENSE = 3         # keep every visual token (full budget)
+TOP_P = 4         # Top-p budgeting, App. A.2: smallest top set with a share p of the scores
 
 PPM = 1_000_000
 
@@ -143,6 +144,26 @@ def budget(m_max: float, n_v: int, mode: int = ADAPTIVE, r_lo_ppm: int = 10_000,
     return min(max(raw, k_lo), k_hi, n_v)
 
 
+def top_p_budget(s: np.ndarray, ratio_ppm: int) -> int:
+    """Top-p budget of App. A.2 (studied with p = 0.10).  The paper does not
+    say over which set the probabilities are normalised; read here as the
+    importance scores of the visual span: K_t is the smallest k whose k
+    largest scores (ranked as in Eq. 3, float32-rounded, ties to the lower
+    index) sum to at least p times the sum of all visual scores.  p is given
+    in parts per million; p <= 0 keeps nothing, p >= 1 keeps every token.
+    """
+    n = len(s)
+    if n == 0 or ratio_ppm <= 0:
+        return 0
+    if ratio_ppm >= PPM:
+        return n
+    s32 = np.asarray(s, dtype=np.float32)
+    order = np.lexsort((np.arange(n), -s32.astype(np.float64)))
+    c = np.cumsum(s32[order].astype(np.float64))
+    target = (ratio_ppm / PPM) * c[-1]
+    return min(int(np.searchsorted(c, target, side="left")) + 1, n)
+
+
 def importance(a: np.ndarray, vis: np.ndarray, heads=None) -> np.ndarray:
     """Importance score of Eq. 2: S_i = (1/H) sum_h A_h(q_t, v_i) over visual i.
 
@@ -222,7 +243,12 @@ def decode_step(q, k, v, vis_start: int, vis_len: int, text_len: int, *,
     a_tau = softmax_tau(z, tau)                              # Eq. 6
     mass, m_mean, m_max = visual_mass(a_tau, vis)            # Eq. 5 + head-max
     _, m_mean1, _ = visual_mass(a1, vis)
-    k_t = budget(m_max, vis_len, mode, r_lo_ppm, r_hi_ppm, ratio_ppm, fixed_k)
+    if mode == TOP_P:
+        if granularity != 0:
+            raise ValueError("the top-p budget is defined for one kept set per sequence")
+        k_t = top_p_budget(importance(a1, vis), ratio_ppm)
+    else:
+        k_t = budget(m_max, vis_len, mode, r_lo_ppm, r_hi_ppm, ratio_ppm, fixed_k)
     if force_k is not None:
         k_t = int(force_k)
 

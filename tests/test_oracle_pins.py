@@ -414,3 +414,39 @@ def test_active_count_per_kv_head():
     assert n.shape == (2,) and act.shape == (2, nv)
     for g in range(2):
         assert n[g] == (s[g].astype(np.float32) > np.float32(0.02)).sum()
+
+
+# ------------------------------------------------------------- top-p budget
+
+def test_top_p_uniform_scores_closed_form():
+    """q = 0: all scores equal, so the top-p set is ceil(p * N_v) tokens (p * N_v
+    not an integer here), the first ones by the tie rule."""
+    q, k, v, vs, nv, tl = _rand_case(61, n_v=20, text=6)
+    for ppm, want in ((130_000, 3), (10_000, 1), (999_000, 20), (560_000, 12)):
+        r = O.decode_step(np.zeros_like(q), k, v, vs, nv, tl, mode=O.TOP_P, ratio_ppm=ppm)
+        assert r["k_t"] == want
+        assert list(r["kept"][0]) == list(range(want))
+
+
+def test_top_p_brute_force_over_subsets():
+    """K is the smallest size of ANY subset of visual tokens whose scores reach a
+    share p of the total (the best subset of a size is its top scores)."""
+    for seed in range(6):
+        q, k, v, vs, nv, tl = _rand_case(70 + seed, n_v=9, text=3, scale_q=3.0)
+        s = O.decode_step(q, k, v, vs, nv, tl)["s"].astype(np.float32).astype(np.float64)
+        for ppm in (50_000, 200_000, 500_000, 900_000):
+            target = ppm / 1e6 * s.sum()
+            want = min(kk for kk in range(1, nv + 1)
+                       if any(sum(s[list(c)]) >= target for c in itertools.combinations(range(nv), kk)))
+            assert O.top_p_budget(s, ppm) == want
+
+
+def test_top_p_limits_and_monotonicity():
+    q, k, v, vs, nv, tl = _rand_case(62, n_v=40, text=5, scale_q=2.0)
+    s = O.decode_step(q, k, v, vs, nv, tl)["s"]
+    assert O.top_p_budget(s, 0) == 0 and O.top_p_budget(s, 1_000_000) == nv
+    ks = [O.top_p_budget(s, ppm) for ppm in range(0, 1_000_001, 50_000)]
+    assert all(a <= b for a, b in zip(ks, ks[1:]))
+    dominant = np.r_[np.full(9, 0.02), 0.5]               # one token holds 0.5 / 0.68 = 74% of the scores
+    assert O.top_p_budget(dominant, 100_000) == 1 and O.top_p_budget(dominant, 730_000) == 1
+    assert O.top_p_budget(dominant, 750_000) == 2
