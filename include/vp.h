@@ -52,7 +52,10 @@ typedef enum {
   VP_ADAPTIVE = 0,    /* K_t = ceil(M_vis,max(tau) * N_v) clamped to [K_lo, K_hi] (Eq. 7, Sec. 5.2) */
   VP_FIXED_RATIO = 1, /* K_t = max(1, ceil(ratio * N_v))   (FastV-VP "Fix Ratio", Table 2)        */
   VP_FIXED_K = 2,     /* K_t = min(fixed_k, N_v)           (Top-k budgeting, App. A.2)             */
-  VP_DENSE = 3        /* K_t = N_v: keep every visual token (full budget)                          */
+  VP_DENSE = 3,       /* K_t = N_v: keep every visual token (full budget)                          */
+  VP_TOP_P = 4        /* K_t = the fewest top-ranked tokens whose S_i sum to >= ratio * sum of all
+                         visual S_i (Top-p budgeting, App. A.2); granularity 0 only; may keep up
+                         to N_v tokens, so kept_cap must be >= max_visual                         */
 } vp_budget_mode;
 
 /* Static shapes, fixed for the life of a context (vp_init). */
@@ -105,7 +108,7 @@ typedef struct {
   float scale;         /* logit scale; 0 means 1/sqrt(D)                                 */
   int32_t r_lo_ppm;    /* ADAPTIVE clamp, parts per million: K_lo = ceil(r_lo*N_v)       */
   int32_t r_hi_ppm;    /*   K_hi = max(K_lo, floor(r_hi*N_v)); e.g. 10000 / 50000 (Sec. 5.2) */
-  int32_t ratio_ppm;   /* FIXED_RATIO ratio, parts per million                           */
+  int32_t ratio_ppm;   /* FIXED_RATIO ratio, or TOP_P share p, parts per million         */
   int32_t fixed_k;     /* FIXED_K budget                                                 */
   int32_t granularity; /* 0: one kept set per sequence, S averaged over all H heads (Eq. 2);
                           1: one kept set per kv-head, S averaged over its G query heads  */

@@ -69,7 +69,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 int32_t max_kept(const vp_budget& bd, int32_t n) {
   if (n <= 0) return 0;
   switch (bd.mode) {
-    case VP_DENSE: return n;
+    case VP_DENSE:
+    case VP_TOP_P: return n;
     case VP_FIXED_K: return bd.fixed_k < n ? (bd.fixed_k < 0 ? 0 : bd.fixed_k) : n;
     case VP_FIXED_RATIO: {
       int64_t k = ceil_div((int64_t)bd.ratio_ppm * n, kPpm);
@@ -87,7 +88,7 @@ int32_t max_kept(const vp_budget& bd, int32_t n) {
 }
 
 bool budget_ok(const vp_budget& bd, std::string* why) {
-  if (bd.mode < VP_ADAPTIVE || bd.mode > VP_DENSE) { *why = "budget.mode out of range"; return false; }
+  if (bd.mode < VP_ADAPTIVE || bd.mode > VP_TOP_P) { *why = "budget.mode out of range"; return false; }
   if (!(bd.tau > 0.f) || !isfinite(bd.tau)) { *why = "budget.tau must be finite and > 0"; return false; }
   if (!(bd.scale >= 0.f) || !isfinite(bd.scale)) { *why = "budget.scale must be finite and >= 0"; return false; }
   if (bd.r_lo_ppm < 0 || bd.r_lo_ppm > kPpm || bd.r_hi_ppm < 0 || bd.r_hi_ppm > kPpm) {
@@ -96,6 +97,7 @@ bool budget_ok(const vp_budget& bd, std::string* why) {
   if (bd.ratio_ppm < 0 || bd.ratio_ppm > kPpm) { *why = "budget.ratio_ppm must lie in [0, 1000000]"; return false; }
   if (bd.fixed_k < 0) { *why = "budget.fixed_k must be >= 0"; return false; }
   if (bd.granularity != 0 && bd.granularity != 1) { *why = "budget.granularity must be 0 or 1"; return false; }
+  if (bd.mode == VP_TOP_P && bd.granularity != 0) { *why = "the top-p budget needs granularity 0"; return false; }
   return true;
 }
 

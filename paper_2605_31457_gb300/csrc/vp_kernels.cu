@@ -52,7 +52,7 @@ constexpr int kGatherTile = 64;           // kept tokens staged per round in k_g
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // an mbarrier wait gives up after 1 s
 
 // Budget modes (numbering of vp_budget_mode in include/vp.h).
-enum { MODE_ADAPTIVE = 0, MODE_FIXED_RATIO = 1, MODE_FIXED_K = 2, MODE_DENSE = 3 };
+enum { MODE_ADAPTIVE = 0, MODE_FIXED_RATIO = 1, MODE_FIXED_K = 2, MODE_DENSE = 3, MODE_TOP_P = 4 };
 
 // ------------------------------------------------------------------ helpers
 
@@ -1290,6 +1290,7 @@ __device__ __forceinline__ int budget_k(const StepParams& p, float m_max, int nv
   if (nv <= 0) return 0;
   switch (p.mode) {
     case MODE_DENSE: return nv;
+    case MODE_TOP_P: return 0;  // decided by the radix select over the score sums
     case MODE_FIXED_K: return max(0, min(p.fixed_k, nv));
     case MODE_FIXED_RATIO: {
       const long long k = ((long long)p.ratio_ppm * nv + 999999) / 1000000;
@@ -1342,12 +1343,17 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   __shared__ int wsum_s[32];
   __shared__ int sh_i[4];
   __shared__ int act_s, act_rank_s[8];  // active-token counts (diagnostics)
+  __shared__ float hsum_s[3][256];      // top-p: score sums per digit
+  __shared__ float vsum_s, vsum_rank_s[8];
 
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
   const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int i = tid; i < 3 * 256; i += NTH) (&hist_s[0][0])[i] = 0;
-  if (tid == 0) act_s = 0;
+  if (tid == 0) { act_s = 0; vsum_s = 0.f; }
+  const bool topp = p.mode == MODE_TOP_P;
+  if (topp)
+    for (int i = tid; i < 3 * 256; i += NTH) (&hsum_s[0][0])[i] = 0.f;
   pdl_wait();
   pdl_trigger();
   const int H = p.H, ns = p.ns;
@@ -1443,10 +1449,11 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
       if (lane == 0) {
         const int K = min(budget_k(p, mx, nv), p.kept_cap);
         sh_i[0] = K;
-        p.kept_count[(int64_t)b * nsel + gsel] = K;
+        if (!topp) p.kept_count[(int64_t)b * nsel + gsel] = K;  // top-p: after the select
         if (gsel == 0 && p.mass_stats) {
           float* ms = p.mass_stats + (int64_t)b * 4;
-          ms[0] = sm / H; ms[1] = mx; ms[2] = s1 / H; ms[3] = (float)K;
+          ms[0] = sm / H; ms[1] = mx; ms[2] = s1 / H;
+          if (!topp) ms[3] = (float)K;
         }
       }
     } else if (gsel == 0) {
@@ -1464,6 +1471,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   unsigned bad = 0;
   const bool diag = p.n_act || p.act_bits;
   int n_on = 0;
+  float vsum = 0.f;  // top-p: this thread's share of the visual score total
   for (int i = i0 + tid; i < i1; i += NTH) {
     const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
     float a = 0.f;
@@ -1494,17 +1502,23 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     const float sc = a * inv_cnt;
     if (!isfinite(sc)) bad = 1;
     key0[i] = __float_as_uint(sc);
+    vsum += sc;
     if (diag && __float_as_uint(sc) > p.act_delta_bits) {  // S_i > delta (Sec. 4.3)
       ++n_on;
       if (p.act_bits) atomicOr(p.act_bits + ((int64_t)b * nsel + gsel) * p.act_words + (i >> 5), 1u << (i & 31));
     }
   }
   if (bad) atomicOr(p.err, ERR_NONFINITE);
-  if (p.n_act) {  // this rank's count, into rank 0's slot
+  if (p.n_act || topp) {  // this rank's count and score total, into rank 0's slots
     n_on = __reduce_add_sync(0xffffffffu, n_on);
+    vsum = warp_sum(vsum);
     if (lane == 0 && n_on) atomicAdd(&act_s, n_on);
+    if (lane == 0 && topp) atomicAdd(&vsum_s, vsum);
     __syncthreads();
-    if (tid == 0) (ncl > 1 ? cluster.map_shared_rank(act_rank_s, 0) : act_rank_s)[rank] = act_s;
+    if (tid == 0) {
+      (ncl > 1 ? cluster.map_shared_rank(act_rank_s, 0) : act_rank_s)[rank] = act_s;
+      (ncl > 1 ? cluster.map_shared_rank(vsum_rank_s, 0) : vsum_rank_s)[rank] = vsum_s;
+    }
   }
   if (ncl > 1) cluster.sync();  // rank 0 now sees every key (and its own K)
   else __syncthreads();
@@ -1515,17 +1529,120 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     for (int r = 0; r < ncl; ++r) n += act_rank_s[r];
     p.n_act[(int64_t)b * nsel + gsel] = n;
   }
-  const int K = sh_i[0];
+  int K = sh_i[0];
   int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
 
   // 4. Radix select of the K-th largest key, 8 bits per pass from the top;
   //    lanes holding the same digit add to the histogram once per warp.  One
   //    barrier per pass: every warp scans the finished histogram itself, and
   //    pass p clears the buffer of pass p - 2 for pass p + 1.
-  const bool take_all = K >= nv;
   uint32_t theta = 0;
   unsigned krem = 0, n_theta = 0;  // keys equal to theta: to keep, in total
-  if (K > 0 && !take_all) {
+  if (topp) {
+    // Top-p budget (App. A.2): the fewest top keys whose scores reach a share
+    // p of the visual total.  Radix select over the score mass: each pass
+    // keeps every digit above the one where the remaining mass is reached.
+    float total = 0.f;
+    for (int r = 0; r < ncl; ++r) total += vsum_rank_s[r];
+    K = 0;
+    if (nv > 0 && p.ratio_ppm >= 1000000) {
+      K = nv;
+    } else if (nv > 0 && p.ratio_ppm > 0) {
+      float need = (float)p.ratio_ppm * 1e-6f * total;  // score mass still to cover
+      unsigned above = 0;                                // keys above the current bucket
+      uint32_t prefix = 0, mask = 0;
+      bool all = false;
+      for (int pass = 0; pass < 4 && !all; ++pass) {
+        const int shift = 24 - 8 * pass;
+        unsigned* hist = hist_s[pass % 3];
+        float* hsum = hsum_s[pass % 3];
+        if (pass >= 2)
+          for (int i = tid; i < 256; i += NTH) { hist_s[(pass + 1) % 3][i] = 0; hsum_s[(pass + 1) % 3][i] = 0.f; }
+        for (int base = 0; base < nv; base += NTH) {
+          const int i = base + tid;
+          const uint32_t kk = i < nv ? key_s[i] : 0u;
+          const bool m = i < nv && (kk & mask) == prefix;
+          const unsigned dg = (kk >> shift) & 255u;
+          const unsigned act = __ballot_sync(0xffffffffu, m);
+          if (act) {
+            const int leader = __ffs(act) - 1;
+            const unsigned d0 = __shfl_sync(0xffffffffu, dg, leader);
+            if (__all_sync(0xffffffffu, !m || dg == d0)) {
+              const float ws = warp_sum(m ? __uint_as_float(kk) : 0.f);
+              if (lane == leader) { atomicAdd(&hist[d0], (unsigned)__popc(act)); atomicAdd(&hsum[d0], ws); }
+            } else if (m) {
+              atomicAdd(&hist[dg], 1u);
+              atomicAdd(&hsum[dg], __uint_as_float(kk));
+            }
+          }
+        }
+        __syncthreads();
+        unsigned cc[8], ctot = 0;
+        float cs[8], stot = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          cc[j] = hist[255 - 8 * lane - j]; ctot += cc[j];
+          cs[j] = hsum[255 - 8 * lane - j]; stot += cs[j];
+        }
+        unsigned cin = ctot;
+        float sin_ = stot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned nc = __shfl_up_sync(0xffffffffu, cin, o);
+          const float ns_ = __shfl_up_sync(0xffffffffu, sin_, o);
+          if (lane >= o) { cin += nc; sin_ += ns_; }
+        }
+        const unsigned cex = cin - ctot;
+        const float sex = sin_ - stot;
+        const bool mine = sex < need && need <= sin_ && ctot > 0;
+        unsigned dsel = 0, cnt_before = 0, cnt = 0;
+        float sum_before = 0.f;
+        if (mine) {
+          // The lane's own running sum may round differently from the scan:
+          // without a digit reaching the mass, its last non-empty digit holds it.
+          unsigned cr = cex;
+          float sr = sex;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (cc[j] > 0) { dsel = 255 - 8 * lane - j; cnt_before = cr; sum_before = sr; cnt = cc[j]; }
+            if (cc[j] > 0 && sr + cs[j] >= need) break;
+            cr += cc[j];
+            sr += cs[j];
+          }
+        }
+        const unsigned found = __ballot_sync(0xffffffffu, mine && cnt > 0);
+        if (!found) { all = true; break; }  // rounding left the mass short: keep every candidate
+        const int src = __ffs(found) - 1;
+        dsel = __shfl_sync(0xffffffffu, dsel, src);
+        cnt_before = __shfl_sync(0xffffffffu, cnt_before, src);
+        sum_before = __shfl_sync(0xffffffffu, sum_before, src);
+        cnt = __shfl_sync(0xffffffffu, cnt, src);
+        above += cnt_before;
+        need -= sum_before;
+        prefix |= dsel << shift;
+        mask |= 255u << shift;
+        if (shift == 0) n_theta = cnt;
+      }
+      if (all) {
+        K = nv;
+      } else {
+        theta = prefix;
+        const float tv = __uint_as_float(theta);
+        unsigned m_eq = tv > 0.f ? (unsigned)ceilf(need / tv) : n_theta;
+        m_eq = max(1u, min(m_eq, n_theta));
+        krem = m_eq;
+        K = (int)(above + m_eq);
+      }
+    }
+    K = min(K, p.kept_cap);
+    if (tid == 0) {
+      p.kept_count[(int64_t)b * nsel + gsel] = K;
+      if (gsel == 0 && p.mass_stats) p.mass_stats[(int64_t)b * 4 + 3] = (float)K;
+    }
+    if (K >= nv) krem = 0;
+  }
+  bool take_all = K >= nv;
+  if (!topp && K > 0 && !take_all) {
     uint32_t prefix = 0, mask = 0;
     krem = (unsigned)K;
     for (int pass = 0; pass < 4; ++pass) {

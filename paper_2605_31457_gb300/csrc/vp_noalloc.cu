@@ -49,7 +49,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 int64_t max_kept(const vp_budget& bd, int64_t n) {
   if (n <= 0) return 0;
   switch (bd.mode) {
-    case VP_DENSE: return n;
+    case VP_DENSE:
+    case VP_TOP_P: return n;
     case VP_FIXED_K: return std::min<int64_t>(std::max<int64_t>(bd.fixed_k, 0), n);
     case VP_FIXED_RATIO: return std::min<int64_t>(std::max<int64_t>(ceil_div((int64_t)bd.ratio_ppm * n, 1000000), 1), n);
     case VP_ADAPTIVE: {
@@ -105,7 +106,7 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
     return fail(VP_ERR_UNSUPPORTED, "vp_decode_step_noalloc: shape not supported");
   if (batch < 0 || batch > c.max_batch) return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: batch outside [0, max_batch]");
   if (!(budget->tau > 0.f) || !isfinite(budget->tau) || !(budget->scale >= 0.f) || !isfinite(budget->scale) ||
-      budget->mode < VP_ADAPTIVE || budget->mode > VP_DENSE || budget->r_lo_ppm < 0 || budget->r_lo_ppm > 1000000 ||
+      budget->mode < VP_ADAPTIVE || budget->mode > VP_TOP_P || (budget->mode == VP_TOP_P && budget->granularity != 0) || budget->r_lo_ppm < 0 || budget->r_lo_ppm > 1000000 ||
       budget->r_hi_ppm < 0 || budget->r_hi_ppm > 1000000 || budget->ratio_ppm < 0 || budget->ratio_ppm > 1000000 ||
       budget->fixed_k < 0 || (budget->granularity != 0 && budget->granularity != 1))
     return fail(VP_ERR_INVALID_ARG, "vp_decode_step_noalloc: malformed budget");

@@ -33,6 +33,7 @@ VP_ADAPTIVE = 0
 VP_FIXED_RATIO = 1
 VP_FIXED_K = 2
 VP_DENSE = 3
+VP_TOP_P = 4
 
 EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
             "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc")

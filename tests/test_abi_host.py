@@ -74,6 +74,8 @@ def test_null_context_and_null_free(lib):
     (dict(mode=2, fixed_k=256), 100, 100),
     (dict(mode=3), 576, 576),
     (dict(), 0, 0),
+    (dict(mode=4, ratio_ppm=100_000), 576, 576),               # TOP_P may keep every token
+    (dict(mode=4, ratio_ppm=100_000, granularity=1), 576, -1),  # TOP_P needs one set per sequence
     (dict(mode=9), 10, -1),
     (dict(tau=0.0), 10, -1),
     (dict(granularity=2), 10, -1),

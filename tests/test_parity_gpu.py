@@ -73,6 +73,11 @@ def test_group_sizes(vp, H, Hkv):
     W.ADAPTIVE_10PCT,
     dict(mode=O.ADAPTIVE, tau=0.4, r_lo_ppm=0, r_hi_ppm=1_000_000),
     dict(mode=O.ADAPTIVE, tau=1.0, r_lo_ppm=0, r_hi_ppm=1_000_000),
+    dict(mode=O.TOP_P, tau=0.1, ratio_ppm=100_000),
+    dict(mode=O.TOP_P, tau=0.1, ratio_ppm=500_000),
+    dict(mode=O.TOP_P, tau=0.1, ratio_ppm=10_000),
+    dict(mode=O.TOP_P, tau=0.1, ratio_ppm=1_000_000),
+    dict(mode=O.TOP_P, tau=0.1, ratio_ppm=0),
 ])
 def test_budget_modes(vp, budget):
     r = small()
@@ -320,4 +325,5 @@ def test_sweep_points_full_size(vp, nv):
     the adaptive budget and 5% / 50% retention (slice and chunk gathers)."""
     r = W.sweep_recipe(nv, W.ADAPTIVE_5PCT)
     rep = {}
-    _device_generated(vp, r, (0, 33, 63), [W.ADAPTIVE_5PCT, W.SWEEP_BUDGETS[1], W.SWEEP_BUDGETS[3]], rep)
+    _device_generated(vp, r, (0, 33, 63), [W.ADAPTIVE_5PCT, W.SWEEP_BUDGETS[1], W.SWEEP_BUDGETS[3],
+                                           dict(mode=O.TOP_P, tau=0.1, ratio_ppm=100_000)], rep)
