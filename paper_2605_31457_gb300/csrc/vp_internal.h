@@ -109,8 +109,9 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   const long long tiles = (max_visual + 31) / 32 + 2LL * ((max_seq + 31) / 32);
   const long long slots = 2LL * num_sms;
   // Split count: minimise (waves of CTAs) x (tiles per CTA + a fixed cost of
-  // about 4 tiles per CTA for its start and its partial), keeping at least 8
-  // tiles per CTA; the smaller count wins a tie.
+  // about 12 tiles per CTA for its start, its pipeline fill and its partial;
+  // the constant was measured across the sweep workloads), keeping at least
+  // 8 tiles per CTA; the smaller count wins a tie.
   long long ns_hi = tiles / 8;
   if (ns_hi > kNsMax) ns_hi = kNsMax;
   if (ns_hi < 1) ns_hi = 1;
@@ -118,7 +119,7 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   double best = 0.0;
   for (long long c = 1; c <= ns_hi; ++c) {
     const double waves = (double)((units * c + slots - 1) / slots);
-    const double cost = waves * ((double)tiles / (double)c + 4.0);
+    const double cost = waves * ((double)tiles / (double)c + 12.0);
     if (c == 1 || cost < best * (1.0 - 1e-9)) { best = cost; ns = c; }
   }
   const long long sel = (long long)batch * (granularity ? Hkv : 1);

@@ -755,6 +755,12 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
 
   if (tid < NW * S) mbar_init(reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + tid, 1);
   mbar_fence_init();
+  // The descriptors are kernel parameters, not outputs of the previous kernel:
+  // fetch them while that kernel finishes.
+  if (tid == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmk)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmv)) : "memory");
+  }
   pdl_wait();
   const int G = p.G, H = p.H;
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
