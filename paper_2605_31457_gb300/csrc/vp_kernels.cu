@@ -761,7 +761,12 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmk)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmv)) : "memory");
   }
-  pdl_wait();
+  // The decode step reads only the call's inputs (q, caches, spans, page
+  // table) until its first workspace write, so its setup and first copies
+  // run before griddepcontrol.wait, while the previous kernel of the stream
+  // (which reads the workspace this kernel writes) finishes.  After the
+  // anchor layer the kept sets come from that kernel: wait first.
+  if (ANCHOR) pdl_wait();
   const int G = p.G, H = p.H;
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
   const int T = sq.nv + sq.tl;
@@ -933,6 +938,7 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   const float ctau = p.inv_tau;
   bool timed_out = false;
   int qc = 0;  // first slot of the tile being read
+  if (!ANCHOR) pdl_wait();  // from here on the workspace is written
 
   for (int j = 0; j < nj; ++j) {
     const int t = warp + NW * j;
@@ -945,20 +951,27 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
     const unsigned kt = smem_u32(ring + ks_ * C::SLOT);
 
     // ---- QK for both 16-row halves of the tile, then refill the K slot
-    float c[2][NT][4];
+    // Even and odd k-steps accumulate separately: two short dependency chains
+    // per 16-row half instead of one long one.
+    float c[2][NT][4], c2[2][NT][4];
 #pragma unroll
     for (int sb = 0; sb < 2; ++sb) {
 #pragma unroll
       for (int nn = 0; nn < NT; ++nn)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) c[sb][nn][e] = 0.f;
+        for (int e = 0; e < 4; ++e) c[sb][nn][e] = c2[sb][nn][e] = 0.f;
 #pragma unroll
       for (int ks = 0; ks < C::KS; ++ks) {
         uint32_t a0, a1, a2, a3;
         ldsm_x4(kt + swz_off<C::HALF_BYTES>(16 * sb + krow, 16 * ks + kcol), a0, a1, a2, a3);
 #pragma unroll
-        for (int nn = 0; nn < NT; ++nn) mma_bf16(c[sb][nn], a0, a1, a2, a3, qfr[nn][ks][0], qfr[nn][ks][1]);
+        for (int nn = 0; nn < NT; ++nn)
+          mma_bf16((ks & 1) ? c2[sb][nn] : c[sb][nn], a0, a1, a2, a3, qfr[nn][ks][0], qfr[nn][ks][1]);
       }
+#pragma unroll
+      for (int nn = 0; nn < NT; ++nn)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) c[sb][nn][e] += c2[sb][nn][e];
     }
     qf = qc + 1;
     issue();
@@ -1360,6 +1373,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   const bool topp = p.mode == MODE_TOP_P;
   if (topp)
     for (int i = tid; i < 3 * 256; i += NTH) (&hsum_s[0][0])[i] = 0.f;
+  const Seq sq = load_seq(p, b, false);  // an input: read before the wait
   pdl_wait();
   pdl_trigger();
   const int H = p.H, ns = p.ns;
@@ -1383,7 +1397,6 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   float4 cx0, cy0, cx1, cy1;
   fetch(warp, lane, cx0, cy0);
   fetch(warp, lane + 32, cx1, cy1);
-  const Seq sq = load_seq(p, b, false);
   const int nv = sq.nv;
   // This rank's slice of the visual tokens; its first logit row is requested
   // now so that it arrives while the statistics are merged (heads up to 32;
