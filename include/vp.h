@@ -200,6 +200,20 @@ vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
  */
 vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t* active_bits);
 
+/* Score kernel of later vp_decode_step calls on this context (an
+ * implementation choice with no counterpart in the paper; results agree
+ * within the documented tolerances either way):
+ *   VP_SCORE_AUTO (default)  the library chooses per call;
+ *   VP_SCORE_MMA             the mma.sync kernels (32-row tiles);
+ *   VP_SCORE_TC              the tcgen05 kernel (128-row tiles, TMEM
+ *                            accumulators): bf16, head_dim 128, G <= 16,
+ *                            pages of at least 8 tokens, a cache layout a
+ *                            tensor descriptor can describe -- a call it
+ *                            cannot serve returns VP_ERR_UNSUPPORTED.
+ * Returns VP_ERR_INVALID_ARG for another value. */
+typedef enum { VP_SCORE_AUTO = 0, VP_SCORE_MMA = 1, VP_SCORE_TC = 2 } vp_score_path;
+vp_status vp_set_score_path(vp_ctx* ctx, int32_t path);
+
 /* Largest K_t the budget can produce for n_visual tokens (the kept_cap a
  * caller must provide); -1 for an invalid budget.  Host only, no CUDA. */
 int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual);

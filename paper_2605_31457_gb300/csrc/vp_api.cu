@@ -32,6 +32,7 @@ struct vp_ctx {
   float diag_delta = 0.f;          // diagnostics (vp_set_diagnostics)
   int32_t* diag_n_act = nullptr;
   uint32_t* diag_bits = nullptr;
+  int32_t score_path = VP_SCORE_AUTO;  // vp_set_score_path
   unsigned* tickets = nullptr;
   unsigned* err = nullptr;
   std::string last_error;
@@ -256,12 +257,12 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   p.mass = mass; p.mass_stats = mass_stats;
   p.z_ws = ctx->z_ws; p.split_st = ctx->split_st; p.split_o = ctx->split_o;
   p.gpart_o = ctx->gpart_o; p.gpart_st = ctx->gpart_st; p.tickets = ctx->tickets; p.err = ctx->err;
-  const vp::Plan pl = vp::make_plan(batch, Hkv, c.head_dim, ctx->num_sms, c.max_visual, c.max_seq, kept_cap,
-                                    budget->granularity);
   p.hp = ctx->lay.hp;
-  p.ns = pl.ns; p.nsp_max = ctx->lay.nsp_max; p.cl = pl.cl;
-  p.nk = pl.nk; p.nk_max = ctx->lay.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice; p.split_w = pl.split_w;
-  vp::encode_kv_maps(p);
+  p.nsp_max = ctx->lay.nsp_max;
+  p.nk_max = ctx->lay.nk_max;
+  if (!vp::plan_step(p, ctx->num_sms, kept_cap, budget->granularity, ctx->score_path))
+    return fail(ctx, VP_ERR_UNSUPPORTED, "vp_decode_step: the tcgen05 score kernel (VP_SCORE_TC) cannot serve this "
+                "call (needs bf16, head_dim 128, G <= 16, pages of >= 8 tokens, a tensor-descriptor layout)");
   p.mt_o = ctx->mt_o; p.mt_st = ctx->mt_st; p.hmax = ctx->hmax;
   if (ctx->diag_n_act || ctx->diag_bits) {
     memcpy(&p.act_delta_bits, &ctx->diag_delta, sizeof(float));
@@ -385,6 +386,15 @@ vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t*
   ctx->diag_delta = delta;
   ctx->diag_n_act = n_act;
   ctx->diag_bits = active_bits;
+  return VP_OK;
+}
+
+vp_status vp_set_score_path(vp_ctx* ctx, int32_t path) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  ctx->last_error.clear();
+  if (path != VP_SCORE_AUTO && path != VP_SCORE_MMA && path != VP_SCORE_TC)
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_set_score_path: path must be VP_SCORE_AUTO, VP_SCORE_MMA or VP_SCORE_TC");
+  ctx->score_path = path;
   return VP_OK;
 }
 

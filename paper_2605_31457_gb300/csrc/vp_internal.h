@@ -36,6 +36,11 @@ struct StepParams {
   CUtensorMap tmk;  // 64-byte aligned type
   CUtensorMap tmv;
   int use_tma;
+  // the same caches in boxes of up to 128 rows, for the tensor-core score
+  // kernel (decode step, bf16, D = 128, at most 16 query heads per kv-head)
+  CUtensorMap tmk2;
+  CUtensorMap tmv2;
+  int use_tc;
   int anchor;  // 1: a layer after the anchor layer -- text plus the given kept set, no selection
   int tpos, gpos, bpos;  // descriptor dimension (1..3) of the token, kv-head and sequence/page axes
   // shapes
@@ -90,6 +95,8 @@ struct StepParams {
 // ---------------------------------------------------------------- host planning
 
 constexpr int kNkMax = 64;    // kept chunks per (sequence, kv-head)
+constexpr int kTcRows = 128;  // rows of a tile of the tensor-core score kernel
+constexpr int kTcMaxBoxes = 384;  // page ids per cache a tensor-core score CTA stages
 constexpr int kNsMax = 256;   // score splits per (sequence, kv-head)
 constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
 
@@ -101,25 +108,36 @@ struct Plan {
   int split_w;  // weight (tiles, text tiles counting 2) of one score split
 };
 
+// tc: the score splits are for the tensor-core kernel (128-row tiles).
 inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, int max_seq, int kept_cap,
-                      int granularity) {
+                      int granularity, bool tc = false) {
   const long long units = (long long)batch * Hkv;
-  // Work of the longest sequence in 32-token tiles (text tiles carry K and V,
-  // so they weigh 2).  Score CTAs are small enough that two fit on an SM.
-  const long long tiles = (max_visual + 31) / 32 + 2LL * ((max_seq + 31) / 32);
+  const int TR = tc ? kTcRows : 32;
+  // Fixed-weight splits sized for the longest sequence (tiles wholly inside
+  // the visual span carry K only and weigh 1, the others K and V and weigh
+  // 2): shorter sequences use fewer splits, so every working score CTA
+  // carries about the same work.
+  long long w_max = 2LL * ((max_seq + TR - 1) / TR) - max_visual / TR;
+  if (w_max < 1) w_max = 1;
+  // Work of the longest sequence in tiles for the split count (32-row tiles:
+  // the visual span counted once more).  Score CTAs are small enough that
+  // two fit on an SM.
+  const long long tiles = tc ? w_max : (max_visual + 31) / 32 + 2LL * ((max_seq + 31) / 32);
   const long long slots = 2LL * num_sms;
-  // Split count: minimise (waves of CTAs) x (tiles per CTA + a fixed cost of
-  // about 12 tiles per CTA for its start, its pipeline fill and its partial;
-  // the constant was measured across the sweep workloads), keeping at least
-  // 8 tiles per CTA; the smaller count wins a tie.
-  long long ns_hi = tiles / 8;
+  // Split count: minimise (waves of CTAs) x (tiles per CTA + a fixed cost per
+  // CTA for its start, its pipeline fill and its partial), keeping a minimum
+  // of work per CTA; the smaller count wins a tie.  The costs were measured
+  // across the sweep workloads: about 12 tiles of 32 rows for the mma.sync
+  // kernel, about 6 weight units of 128 rows for the tensor-core kernel.
+  long long ns_hi = tiles / (tc ? 2 : 8);
   if (ns_hi > kNsMax) ns_hi = kNsMax;
   if (ns_hi < 1) ns_hi = 1;
+  const double fixed = tc ? 6.0 : 12.0;
   long long ns = 1;
   double best = 0.0;
   for (long long c = 1; c <= ns_hi; ++c) {
     const double waves = (double)((units * c + slots - 1) / slots);
-    const double cost = waves * ((double)tiles / (double)c + 12.0);
+    const double cost = waves * ((double)tiles / (double)c + fixed);
     if (c == 1 || cost < best * (1.0 - 1e-9)) { best = cost; ns = c; }
   }
   const long long sel = (long long)batch * (granularity ? Hkv : 1);
@@ -143,10 +161,6 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   // Small kept sets of few sequences: one CTA per 16 output dimensions, so
   // that the whole gather is one short wave; otherwise one CTA per chunk.
   const int gslice = kept_cap <= 256 && units * (D / 16) <= slots ? 1 : 0;
-  // Fixed-weight splits sized for the longest sequence: shorter ones use
-  // fewer splits, so every working score CTA carries about the same work.
-  long long w_max = 2LL * ((max_seq + 31) / 32) - max_visual / 32;
-  if (w_max < 1) w_max = 1;
   const int split_w = (int)((w_max + ns - 1) / ns);
   return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), gslice, split_w};
 }
@@ -165,10 +179,11 @@ inline WsLayout ws_layout(int batch, int H, int Hkv, int D, int max_visual, int 
   w.hp = (H + 3) / 4 * 4;
   w.nk_max = kNkMax;
   w.nsp_max = 1;
-  for (int bb = 1; bb <= batch; ++bb) {
-    const Plan pl = make_plan(bb, Hkv, D, num_sms, max_visual, max_seq, 0, 0);
-    if (pl.ns > w.nsp_max) w.nsp_max = pl.ns;
-  }
+  for (int bb = 1; bb <= batch; ++bb)
+    for (int tc = 0; tc < 2; ++tc) {
+      const Plan pl = make_plan(bb, Hkv, D, num_sms, max_visual, max_seq, 0, 0, tc != 0);
+      if (pl.ns > w.nsp_max) w.nsp_max = pl.ns;
+    }
   const size_t B = (size_t)batch, G = (size_t)(H / Hkv);
   size_t off = 0;
   w.o_tickets = off; off = ws_round(off + B * Hkv * 4);
@@ -196,6 +211,42 @@ cudaError_t configure_kernels(int max_visual, int H, int nsp_max);
 // Fills p.tmk / p.tmv / p.use_tma for a bf16 cache whose layout a 4-D tensor
 // descriptor can describe without reaching past the caller's memory; leaves
 // use_tma = 0 otherwise (the score kernel then copies rows one by one).
+// With p.use_tc set on entry (a plan made for the tensor-core kernel) it also
+// fills p.tmk2 / p.tmv2 and keeps use_tc only if that kernel can run.
 void encode_kv_maps(StepParams& p);
+// The tensor-core score kernel's shape conditions (decode step, bf16, D = 128,
+// at most 16 query heads per kv-head, pages of at least 8 rows).
+inline bool tc_eligible(int dtype, int D, int G, int paged, int page_size) {
+  return dtype == 0 && D == 128 && G >= 1 && G <= 16 && (!paged || page_size >= 8);
+}
+
+// Launch plan and copy descriptors of a decode step (p's shapes, inputs and
+// dtype set): the tensor-core score kernel where it can run and pays off,
+// otherwise the mma.sync kernels with their own split count.  The
+// tensor-core kernel moves 128-row tiles and holds TMEM, so a CTA starts
+// later: it is chosen when every (sequence, kv-head) carries at least 32
+// weight units of 128-row tiles (about 2000 cache rows) and the call has
+// work for many such CTAs (measured: below either bound the mma.sync
+// kernel was faster, above both the tensor-core kernel).
+// path: 0 the choice above, 1 never the tensor-core kernel, 2 only it
+// (false when it cannot serve the call).
+inline bool plan_step(StepParams& p, int num_sms, int kept_cap, int granularity, int path = 0) {
+  const long long w_tc = 2LL * ((p.max_seq + kTcRows - 1) / kTcRows) - p.max_visual / kTcRows;
+  const bool eligible = tc_eligible(p.dtype, p.D, p.G, p.paged, p.page_size);
+  const bool tc = path == 2 ? eligible
+                            : path == 0 && eligible && w_tc >= 32 && (long long)p.B * p.Hkv * w_tc >= 16LL * num_sms;
+  if (path == 2 && !tc) return false;
+  for (int pass = 0; pass < 2; ++pass) {
+    const bool want = tc && pass == 0;
+    const Plan pl = make_plan(p.B, p.Hkv, p.D, num_sms, p.max_visual, p.max_seq, kept_cap, granularity, want);
+    p.ns = pl.ns; p.cl = pl.cl; p.nk = pl.nk; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice;
+    p.split_w = pl.split_w;
+    p.use_tc = want ? 1 : 0;
+    encode_kv_maps(p);
+    if (p.use_tc || !want) return true;
+    if (path == 2) return false;
+  }
+  return true;
+}
 
 }  // namespace vp

@@ -1137,6 +1137,534 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
 }
 
 // ---------------------------------------------------------------------------
+// k_score_tc (bf16, D = 128, up to 16 query heads per kv-head): the decode
+// step's score kernel on the fifth-generation tensor cores.  Grid (splits,
+// Hkv, B) with the splits cut in 128-row tiles; 192 threads in three roles:
+//   warp 0     (one lane) copies each tile's K, and its V where the tile holds
+//              rows outside the visual span, with 4-D bulk-tensor copies into
+//              a ring of three 32 KB slots (128-byte swizzle);
+//   warp 1     holds 64 TMEM columns and (one lane) issues tcgen05.mma:
+//              S = K q^T (M = 128 tokens, N = 16 heads, K = 128 dimensions)
+//              into one of two S buffers, and O += V^T P^T (M = 128
+//              dimensions, N = 16 heads, K = 128 tokens) into the O buffer,
+//              each completion signalled by tcgen05.commit on an mbarrier;
+//   warps 2-5  (one thread per token row; for O, per dimension) read S with
+//              tcgen05.ld, write the visual logits, keep the visual
+//              statistics per thread and turn text logits into probabilities
+//              P = exp2(z - M_ref) for the P.V product.
+// M_ref, a head's text reference maximum, is raised only when a logit passes
+// it by more than theta = min(8, 64 tau) (log2 units), so that P and the
+// tempered sums stay finite; the O accumulator and the sums are then
+// rescaled.  Most tiles need no exchange between the threads.  The split's
+// partial has the meaning of the other score kernels' partials.
+// Waits are bounded: a thread whose wait gives up stops its work, still
+// passes every barrier of its group, and the error word reports the timeout.
+// ---------------------------------------------------------------------------
+constexpr int kTcSlots = 3;  // ring slots of the kernel as launched (two CTAs per SM)
+constexpr int kTcThreads = 192;
+
+template <int NS>
+struct TcCfgT {
+  static constexpr int SLOTS = NS;
+  static constexpr int HALF = kTcRows * 128;           // 128 rows x 64 dimensions, swizzled
+  static constexpr int SLOT = 2 * HALF;                // a 128 x 128 tile of K or of V
+  static constexpr int QHALF = 16 * 128;               // 16 rows x 64 elements
+  static constexpr int OFF_Q = NS * SLOT;              // q: 16 heads x 128 dimensions
+  static constexpr int OFF_P = OFF_Q + 2 * QHALF;      // P^T: 2 buffers of 16 heads x 128 tokens
+  static constexpr int PBUF = 2 * QHALF;
+  static constexpr int OFF_BAR = OFF_P + 2 * PBUF;
+  static constexpr int NBAR = 2 * NS + 9;              // full, empty, s_full, s_free, p_full, pv_done, mma_done
+  static constexpr int OFF_PG = OFF_BAR + (NBAR * 8 + 15) / 16 * 16;
+  static constexpr int OFF_RED = OFF_PG + 2 * kTcMaxBoxes * 4;  // float [4][16]: new text maxima
+  static constexpr int OFF_TMEM = OFF_RED + 4 * 16 * 4;
+  // The partial's reductions, float [4][16][6], take the P buffers once every
+  // P.V product is complete.
+  static_assert(4 * 16 * 6 * 4 <= 2 * PBUF, "reduction buffer fits the P buffers");
+  static constexpr size_t SMEM = 1024 + (size_t)OFF_TMEM + 16;
+  static_assert(SLOT % 1024 == 0 && OFF_Q % 1024 == 0 && OFF_P % 1024 == 0, "swizzle atoms stay aligned");
+};
+using TcCfg = TcCfgT<kTcSlots>;
+
+// Shared-memory matrix descriptor of a 128-byte-swizzled operand (sm_100
+// layout: start, leading and stride byte offsets in 16-byte units, version 1).
+__device__ __forceinline__ uint64_t umma_desc(unsigned addr, unsigned lbo, unsigned sbo) {
+  return (uint64_t)((addr >> 4) & 0x3fffu) | ((uint64_t)((lbo >> 4) & 0x3fffu) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3fffu) << 32) | (1ull << 46) | (2ull << 61);
+}
+// Instruction descriptor: bf16 x bf16 -> f32, M = 128, N = 16; A K-major or
+// MN-major, B K-major.
+__host__ __device__ constexpr uint32_t umma_idesc(int a_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)(16 >> 3) << 17) |
+         ((uint32_t)(128 >> 4) << 24);
+}
+__device__ __forceinline__ void umma(unsigned d, uint64_t a, uint64_t b, uint32_t id, bool acc) {
+  asm volatile("{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+               ::"r"(d), "l"(a), "l"(b), "r"(id), "r"((int)acc) : "memory");
+}
+// Arrives on the mbarrier once this thread's earlier tensor-core operations are complete.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
+__device__ __forceinline__ void tmem_ld16(unsigned taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_st16(unsigned taddr, const float (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n"
+      ::"r"(taddr), "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+        "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+        "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+        "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+        "r"(__float_as_uint(v[15]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
+// Barrier of the four softmax warps (named barrier 1); the second form also
+// counts the threads whose predicate is true.
+__device__ __forceinline__ void wg_sync() { asm volatile("bar.sync 1, 128;\n" ::: "memory"); }
+__device__ __forceinline__ int wg_sync_count(bool pred) {
+  int n;
+  asm volatile("{\n .reg .pred p;\n setp.ne.b32 p, %1, 0;\n bar.red.popc.u32 %0, 1, 128, p;\n}\n"
+               : "=r"(n) : "r"((int)pred) : "memory");
+  return n;
+}
+
+// The 128-row tiles of one split.  Tiles [v0, v1) lie wholly inside the
+// visual span (K only, weight 1); every other tile carries text or padding
+// rows (K and V, weight 2).  Split s owns tiles [u0, u0 + n), a fixed weight
+// per split as in tma_split.
+struct TcRange {
+  int u0, n, v0, v1;
+  __device__ __forceinline__ bool pure(int i) const { return u0 + i >= v0 && u0 + i < v1; }
+};
+__device__ __forceinline__ TcRange tc_split(const Seq& sq, int s, int ns, int split_w) {
+  const int T = sq.nv + sq.tl;
+  const int NTl = (T + kTcRows - 1) / kTcRows;
+  TcRange r;
+  r.v0 = (sq.vs + kTcRows - 1) / kTcRows;
+  r.v1 = max(r.v0, min(NTl, (sq.vs + sq.nv) / kTcRows));
+  const int W = 2 * NTl - (r.v1 - r.v0);
+  const int per = max(split_w, (W + ns - 1) / ns);
+  auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
+    if (w <= 2 * r.v0) return (w + 1) / 2;
+    if (w <= r.v0 + r.v1) return w - r.v0;
+    return (w + (r.v1 - r.v0) + 1) / 2;
+  };
+  r.u0 = tile_of(min(W, s * per));
+  r.n = tile_of(min(W, (s + 1) * per)) - r.u0;
+  return r;
+}
+
+template <int GM, int NS = kTcSlots>
+__global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const __grid_constant__ StepParams p) {
+  using C = TcCfgT<NS>;
+  constexpr int D = 128, S = NS;
+  constexpr uint32_t kIdQK = umma_idesc(0), kIdPV = umma_idesc(1);
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  unsigned char* smem = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);  // [S] a slot's copies landed
+  uint64_t* empty = full + S;                                        // [S] a slot's tile was read
+  uint64_t* s_full = full + 2 * S;                                   // [2] S buffer written
+  uint64_t* s_free = s_full + 2;                                     // [2] S buffer read (128 arrivals)
+  uint64_t* p_full = s_full + 4;                                     // [2] P buffer written (128 arrivals)
+  uint64_t* pv_done = s_full + 6;                                    // [2] P.V of that P buffer complete
+  uint64_t* mma_done = s_full + 8;                                   // every tensor-core operation complete
+  int* kpg = reinterpret_cast<int*>(smem + C::OFF_PG);
+  int* vpg = kpg + kTcMaxBoxes;
+  float (*red)[16] = reinterpret_cast<float (*)[16]>(smem + C::OFF_RED);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_TMEM);
+
+  if (tid == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(full + i, 1);
+      mbar_init(empty + i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(s_full + i, 1);
+      mbar_init(s_free + i, 128);
+      mbar_init(p_full + i, 128);
+      mbar_init(pv_done + i, 1);
+    }
+    mbar_init(mma_done, 1);
+    mbar_fence_init();
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmk2)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmv2)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 64;\n" ::"r"(smem_u32(tmem_slot))
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+  }
+  // Everything up to the first workspace write reads only the call's inputs,
+  // so it runs before griddepcontrol.wait (see k_score_tma).
+  const int G = p.G, H = p.H;
+  const Seq sq = load_seq(p, b, s == 0 && g == 0);
+  const int T = sq.nv + sq.tl;
+  const TcRange tr = tc_split(sq, s, p.ns, p.split_w);
+  const int R = p.paged ? min(kTcRows, p.page_size) : kTcRows;  // rows per copied box
+  const int nb = kTcRows / R;
+  int n = tr.n;
+  unsigned err = 0;
+  if (p.paged) {
+    if (n * nb > kTcMaxBoxes) {  // the host plan keeps every split below this
+      err |= ERR_PAGE;
+      n = 0;
+    }
+    for (int i = tid; i < n * nb; i += kTcThreads) {
+      const int t = i / nb, pos = (tr.u0 + t) * kTcRows + (i % nb) * R;
+      kpg[i] = pos < T ? tma_page(p.k, p, b, pos) : -2;
+      vpg[i] = (pos < T && !tr.pure(t)) ? tma_page(p.v, p, b, pos) : -2;
+    }
+  }
+  if (warp >= 2) {  // q of the kv-head's query heads, rows past G zero, K-major and swizzled
+    const uint32_t* qb = reinterpret_cast<const uint32_t*>(reinterpret_cast<const __nv_bfloat16*>(p.q) +
+                                                           ((int64_t)b * H + g * G) * D);
+    for (int i = tid - 64; i < 16 * (D / 8); i += 128) {
+      const int h = i / (D / 8), c = i % (D / 8);  // 16-byte piece c (dimensions 8c .. 8c + 7)
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (h < G) {
+        const uint32_t* src = qb + h * (D / 2) + 4 * c;
+        v = make_uint4(__ldg(src), __ldg(src + 1), __ldg(src + 2), __ldg(src + 3));
+      }
+      *reinterpret_cast<uint4*>(smem + C::OFF_Q + (c >> 3) * C::QHALF + h * 128 + (((c & 7) ^ (h & 7)) << 4)) = v;
+    }
+    fence_proxy_async();  // read by the tensor core
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const unsigned tmem = *tmem_slot;  // columns [0,16) and [16,32): S buffers; [32,48): O
+  bool timed_out = false;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ copies
+    // Pieces in the order the tensor cores read them: K of tile i, then V of
+    // the text tile before it (its P.V follows tile i's QK).  Lane 0 arms the
+    // slot's barrier; lane 2x + hh copies half hh of box x.
+    int q = 0;  // pieces issued
+    auto issue = [&](int i, int part) {
+      const int sl = q % S;
+      if (!__all_sync(0xffffffffu, mbar_wait(empty + sl, ((q / S) & 1) ^ 1))) return false;
+      const int u = tr.u0 + i;
+      const int* pg = part ? vpg : kpg;
+      bool live = false, bad = false;
+      int base = b, row = 0;
+      const int x = lane >> 1, hh = lane & 1;
+      if (x < nb) {
+        const int pos = u * kTcRows + x * R;
+        if (pos < T) {
+          if (p.paged) {
+            base = pg[i * nb + x];
+            bad = base < 0;
+            row = pos & (p.page_size - 1);
+          } else {
+            row = pos;
+          }
+          live = !bad;
+        }
+      }
+      if (bad) err |= ERR_PAGE;
+      const unsigned n_live = __popc(__ballot_sync(0xffffffffu, live));  // live halves
+      if (lane == 0) mbar_expect_tx(full + sl, n_live * (unsigned)R * 128u);
+      __syncwarp();
+      if (live) {
+        auto crd = [&](int axis) { return axis == p.tpos ? row : axis == p.gpos ? g : base; };
+        tma_load_4d(smem_u32(smem + sl * C::SLOT) + hh * C::HALF + x * R * 128, part ? &p.tmv2 : &p.tmk2, 64 * hh,
+                    crd(1), crd(2), crd(3), full + sl);
+      }
+      ++q;
+      return true;
+    };
+    {
+      int pend = -1;
+      for (int i = 0; i < n && !timed_out; ++i) {
+        if (!issue(i, 0) || (pend >= 0 && !issue(pend, 1))) { timed_out = true; break; }
+        pend = tr.pure(i) ? -1 : i;
+      }
+      if (!timed_out && pend >= 0 && !issue(pend, 1)) timed_out = true;
+      // Copies still in flight (only after a timeout can any be unread) land
+      // before the CTA's shared memory is released.
+      for (int k = max(0, q - S); k < q; ++k) mbar_wait(full + k % S, (k / S) & 1);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------ tensor cores
+    // Tile i's QK is issued before the P.V of the previous text tile, so that
+    // the softmax threads find S(i) ready when they finish that tile's P.
+    // Every lane waits (and zeroes stale V rows); the warp leaves the loop
+    // together when any lane's wait gives up.
+    auto wait_all = [&](uint64_t* bar, unsigned parity) { return __all_sync(0xffffffffu, mbar_wait(bar, parity)); };
+    int q = 0, j = 0;        // pieces read, text tiles multiplied
+    int pend = -1, pq = 0;   // text tile whose P.V is due, and its V piece (read after K of the next tile)
+    auto pv = [&]() {        // the P.V product of text tile `pend`
+      const int sv = pq % S, pb = j & 1;
+      if (!wait_all(full + sv, (pq / S) & 1)) return false;
+      // V rows past the cache or of an unmapped page hold stale bytes: zero
+      // them (their probabilities are 0, but 0 x NaN is not).
+      const int p0 = (tr.u0 + pend) * kTcRows;
+      bool stale = p0 + kTcRows > T;
+      if (p.paged)
+        for (int x = 0; x < nb; ++x) stale |= vpg[pend * nb + x] < 0;
+      if (stale) {
+        unsigned char* vt = smem + sv * C::SLOT;
+        for (int r = lane; r < kTcRows; r += 32) {
+          if (p0 + r < T && !(p.paged && vpg[pend * nb + r / R] < 0)) continue;
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            *reinterpret_cast<uint4*>(vt + (c >> 3) * C::HALF + r * 128 + (c & 7) * 16) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async();
+      }
+      __syncwarp();
+      if (!wait_all(p_full + pb, (j >> 1) & 1)) return false;
+      tc_fence_after();
+      if (lane == 0) {
+        const unsigned vb = smem_u32(smem + sv * C::SLOT), pbs = smem_u32(smem + C::OFF_P + pb * C::PBUF);
+#pragma unroll
+        for (int ks = 0; ks < kTcRows / 16; ++ks)
+          umma(tmem + 32, umma_desc(vb + ks * 2048, C::HALF, 1024),
+               umma_desc(pbs + (ks >> 2) * C::QHALF + (ks & 3) * 32, 16, 1024), kIdPV, j > 0 || ks > 0);
+        umma_commit(pv_done + pb);
+        umma_commit(empty + sv);
+      }
+      __syncwarp();
+      ++j;
+      pend = -1;
+      return true;
+    };
+    for (int i = 0; i < n; ++i) {
+      const int sb = i & 1, sk = q % S;
+      if (!wait_all(full + sk, (q / S) & 1) || !wait_all(s_free + sb, ((i >> 1) & 1) ^ 1)) {
+        timed_out = true;
+        break;
+      }
+      tc_fence_after();
+      if (lane == 0) {
+        const unsigned kb = smem_u32(smem + sk * C::SLOT), qs = smem_u32(smem + C::OFF_Q);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks)
+          umma(tmem + 16 * sb, umma_desc(kb + (ks >> 2) * C::HALF + (ks & 3) * 32, 16, 1024),
+               umma_desc(qs + (ks >> 2) * C::QHALF + (ks & 3) * 32, 16, 1024), kIdQK, ks > 0);
+        umma_commit(s_full + sb);
+        umma_commit(empty + sk);
+      }
+      __syncwarp();
+      ++q;
+      if (pend >= 0) {
+        pq = q++;
+        if (!pv()) { timed_out = true; break; }
+      }
+      if (!tr.pure(i)) pend = i;
+    }
+    if (!timed_out && pend >= 0) {
+      pq = q++;
+      if (!pv()) timed_out = true;
+    }
+    if (lane == 0) umma_commit(mma_done);  // after every operation issued above
+    __syncwarp();
+    if (!mbar_wait(mma_done, 0)) timed_out = true;
+  } else {
+    // -------------------------------------------- softmax (one row each)
+    const int wq = warp & 3;                     // TMEM lanes [32 wq, 32 wq + 32)
+    const int r = wq * 32 + lane;                // token row of a tile; dimension of O
+    const unsigned taddr = tmem + ((unsigned)(wq * 32) << 16);
+    const float inv_tau = p.inv_tau, theta = fminf(8.f, 64.f / inv_tau);
+    float mv[GM], l1v[GM], ltv[GM], mref[GM], l1t[GM], ltt[GM];
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      mv[h] = mref[h] = -CUDART_INF_F;
+      l1v[h] = ltv[h] = l1t[h] = ltt[h] = 0.f;
+    }
+    float* zbase = p.z_ws + (int64_t)b * p.max_visual * p.hp + g * G;
+    const bool zvec = (G & 3) == 0;
+    bool dead = false;  // a wait of this thread gave up: skip the work, keep the barriers
+    pdl_wait();         // from here on the workspace is written
+    int j = 0;          // text tiles seen
+    for (int i = 0; i < n; ++i) {
+      const int u = tr.u0 + i, sb = i & 1;
+      float sv[16];
+      if (!dead && mbar_wait(s_full + sb, (i >> 1) & 1)) {
+        tc_fence_after();
+        tmem_ld16(taddr + 16 * sb, sv);
+      } else {
+        dead = true;
+#pragma unroll
+        for (int h = 0; h < 16; ++h) sv[h] = 0.f;
+      }
+      tc_fence_before();
+      mbar_arrive(s_free + sb);
+      const int pos = u * kTcRows + r;
+      bool valid = !dead && pos < T;
+      if (valid && p.paged) valid = kpg[i * nb + r / R] >= 0;
+      const bool vis = valid && (unsigned)(pos - sq.vs) < (unsigned)sq.nv;
+      const bool txt = valid && !vis;
+#pragma unroll
+      for (int h = 0; h < GM; ++h) sv[h] *= p.c_log2;
+      if (vis) {
+        float* zr = zbase + (int64_t)(pos - sq.vs) * p.hp;
+        if (zvec) {
+#pragma unroll
+          for (int h = 0; h < GM; h += 4)
+            if (h < G) *reinterpret_cast<float4*>(zr + h) = make_float4(sv[h], sv[h + 1], sv[h + 2], sv[h + 3]);
+        } else {
+#pragma unroll
+          for (int h = 0; h < GM; ++h)
+            if (h < G) zr[h] = sv[h];
+        }
+#pragma unroll
+        for (int h = 0; h < GM; ++h) {
+          if (h >= G) continue;
+          const float z = sv[h];
+          if (z > mv[h]) {
+            l1v[h] = fmaf(l1v[h], exp2_rel(mv[h], z), 1.f);
+            ltv[h] = fmaf(ltv[h], exp2_tau(mv[h], z, inv_tau), 1.f);
+            mv[h] = z;
+          } else {
+            l1v[h] += fexp2(z - mv[h]);
+            ltv[h] += fexp2((z - mv[h]) * inv_tau);
+          }
+        }
+      }
+      if (tr.pure(i)) continue;
+      // ---- text rows: raise M_ref where a logit passes it by more than theta
+      bool need = false;
+#pragma unroll
+      for (int h = 0; h < GM; ++h) need |= txt && h < G && sv[h] > mref[h] + theta;
+      if (wg_sync_count(need)) {
+#pragma unroll
+        for (int h = 0; h < GM; ++h) {
+          const float m = warp_max(txt && h < G ? sv[h] : -CUDART_INF_F);
+          if (lane == 0) red[wq][h] = m;
+        }
+        wg_sync();
+        float f[GM];
+#pragma unroll
+        for (int h = 0; h < GM; ++h) {
+          const float mn = fmaxf(mref[h], fmaxf(fmaxf(red[0][h], red[1][h]), fmaxf(red[2][h], red[3][h])));
+          f[h] = exp2_rel(mref[h], mn);
+          l1t[h] *= f[h];
+          ltt[h] *= exp2_tau(mref[h], mn, inv_tau);
+          mref[h] = mn;
+        }
+        wg_sync();  // red is read before its next use
+        if (j > 0 && !dead) {
+          // O holds the products of text tiles 0 .. j - 1: rescale it once the last is complete.
+          if (mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1)) {
+            tc_fence_after();
+            float o[16];
+            tmem_ld16(taddr + 32, o);
+#pragma unroll
+            for (int h = 0; h < GM; ++h) o[h] *= f[h];
+            tmem_st16(taddr + 32, o);
+          } else {
+            dead = true;
+          }
+        }
+      }
+      // ---- probabilities, into P^T (K-major, swizzled) for the P.V product
+      __nv_bfloat16 pr[16];
+#pragma unroll
+      for (int h = 0; h < 16; ++h) {
+        float pe = 0.f;
+        if (h < GM && h < G && txt) {
+          pe = fexp2(sv[h] - mref[h]);
+          l1t[h] += pe;
+          ltt[h] += fexp2((sv[h] - mref[h]) * inv_tau);
+        }
+        pr[h] = __float2bfloat16_rn(pe);
+      }
+      const int pb = j & 1;
+      if (j >= 2 && !dead && !mbar_wait(pv_done + pb, ((j >> 1) & 1) ^ 1)) dead = true;  // buffer free
+      unsigned char* pt = smem + C::OFF_P + pb * C::PBUF + (r >> 6) * C::QHALF + (r & 7) * 2;
+#pragma unroll
+      for (int h = 0; h < 16; ++h)
+        *reinterpret_cast<__nv_bfloat16*>(pt + h * 128 + ((((r & 63) >> 3) ^ (h & 7)) << 4)) = pr[h];
+      fence_proxy_async();
+      tc_fence_before();
+      mbar_arrive(p_full + pb);
+      ++j;
+    }
+    // ---- the split's partial: text output, then statistics
+    float o[16];
+#pragma unroll
+    for (int h = 0; h < 16; ++h) o[h] = 0.f;
+    if (j > 0 && !dead) {
+      if (mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1)) {
+        tc_fence_after();
+        tmem_ld16(taddr + 32, o);
+      } else {
+        dead = true;
+      }
+    }
+    pdl_trigger();
+    float (*red6)[16][6] = reinterpret_cast<float (*)[16][6]>(smem + C::OFF_P);
+#pragma unroll
+    for (int h = 0; h < GM; ++h) {
+      const float M = warp_max(mv[h]);
+      const float a1 = warp_sum(l1v[h] * exp2_rel(mv[h], M)), at = warp_sum(ltv[h] * exp2_tau(mv[h], M, inv_tau));
+      const float c1 = warp_sum(l1t[h]), ct = warp_sum(ltt[h]);
+      if (lane == 0) {
+        red6[wq][h][0] = M; red6[wq][h][1] = a1; red6[wq][h][2] = at;
+        red6[wq][h][3] = c1; red6[wq][h][4] = ct;
+      }
+    }
+    wg_sync();
+    const int64_t rec0 = ((int64_t)b * H + g * G) * p.nsp_max + s;  // split slot of head 0
+    if (r < G) {
+      const int h = r;
+      float M = -CUDART_INF_F;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) M = fmaxf(M, red6[w][h][0]);
+      float a1 = 0.f, at = 0.f, c1 = 0.f, ct = 0.f;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        a1 = fmaf(red6[w][h][1], exp2_rel(red6[w][h][0], M), a1);
+        at = fmaf(red6[w][h][2], exp2_tau(red6[w][h][0], M, inv_tau), at);
+        c1 += red6[w][h][3];
+        ct += red6[w][h][4];
+      }
+      float mt = -CUDART_INF_F;
+#pragma unroll
+      for (int hh = 0; hh < GM; ++hh)
+        if (hh == h) mt = mref[hh];
+      float4* rec = reinterpret_cast<float4*>(p.split_st + (rec0 + (int64_t)h * p.nsp_max) * ST_N);
+      rec[0] = make_float4(mt, c1, ct, 0.f);  // ST_MT, ST_L1T, ST_LTT
+      rec[1] = make_float4(M, a1, at, 0.f);   // ST_MV, ST_L1V, ST_LTV
+    }
+#pragma unroll
+    for (int h = 0; h < GM; ++h)
+      if (h < G) p.split_o[(rec0 + (int64_t)h * p.nsp_max) * D + r] = o[h];
+    if (dead) timed_out = true;
+  }
+  if (timed_out) err |= ERR_TIMEOUT;
+  if (err) atomicOr(p.err, err);
+  // Teardown: every copy has landed and every tensor-core operation is
+  // complete (warps 0 and 1 waited for them, bounded); free the columns.
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 64;\n" ::"r"(tmem) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
 // k_score_f32 (fp32 caches): lane-per-token dot products on the FMA pipes,
 // lane-per-dimension P.V; the same partials as k_score_mma.
 // ---------------------------------------------------------------------------
@@ -2523,6 +3051,10 @@ size_t tma_smem() { return TmaCfg<D, NT, kTmaWarps, tma_slots<D>()>::SMEM; }
 template <int D>
 cudaError_t launch_score_d(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.ns, p.Hkv, p.B);
+  if (D == 128 && p.use_tc && !p.anchor) {
+    if (p.G <= 8) return launch_ex(k_score_tc<8>, grid, dim3(kTcThreads), TcCfg::SMEM, st, 1, p);
+    return launch_ex(k_score_tc<16>, grid, dim3(kTcThreads), TcCfg::SMEM, st, 1, p);
+  }
   if (p.dtype == 0 && p.use_tma) {
     constexpr int NW = kTmaWarps, S = tma_slots<D>();
     if (p.anchor) {
@@ -2570,6 +3102,8 @@ cudaError_t set_smem(void (*kernel)(StepParams), size_t bytes) {
 cudaError_t configure_fixed_kernels() {
   cudaError_t e = cudaSuccess;
 #define VP_SET(kernel, bytes) if (e == cudaSuccess) e = set_smem(kernel, bytes)
+  VP_SET((k_score_tc<8>), (TcCfg::SMEM));
+  VP_SET((k_score_tc<16>), (TcCfg::SMEM));
   VP_SET((k_gather_mma<128, 1>), (GmCfg<128, 1>::SMEM));
   VP_SET((k_gather_mma<128, 2>), (GmCfg<128, 2>::SMEM));
   VP_SET((k_gather_mma<64, 1>), (GmCfg<64, 1>::SMEM));
@@ -2659,9 +3193,10 @@ EncodeTiledFn encode_fn() {
 }
 
 // 4-D descriptor of one cache: dims {D, token, kv-head, sequence or page}, the
-// last three ordered by increasing stride.  Returns false for a layout whose
-// extent along the token axis cannot be bounded by the caller's memory.
-bool encode_one(const KvView& kv, const StepParams& p, CUtensorMap* map, int* tpos, int* gpos, int* bpos) {
+// last three ordered by increasing stride, boxes of 64 dimensions x R rows.
+// Returns false for a layout whose extent along the token axis cannot be
+// bounded by the caller's memory.
+bool encode_one(const KvView& kv, const StepParams& p, CUtensorMap* map, int* tpos, int* gpos, int* bpos, int R) {
   EncodeTiledFn fn = encode_fn();
   if (!fn || !kv.data) return false;
   struct Ax { int64_t stride, size; int id; };  // id: 0 token, 1 kv-head, 2 sequence / page
@@ -2687,7 +3222,6 @@ bool encode_one(const KvView& kv, const StepParams& p, CUtensorMap* map, int* tp
   for (int i = 0; i < 3; ++i)
     if (!p.paged && ax[i].id == 0 && ax[i].size > p.max_seq) dims[i + 1] = (cuuint64_t)p.max_seq;
   const cuuint64_t strides[3] = {(cuuint64_t)ax[0].stride * 2, (cuuint64_t)ax[1].stride * 2, (cuuint64_t)ax[2].stride * 2};
-  const int R = p.paged ? (p.page_size < kTmaTile ? p.page_size : kTmaTile) : kTmaTile;
   cuuint32_t box[4] = {64, 1, 1, 1};
   cuuint32_t estr[4] = {1, 1, 1, 1};
   for (int i = 0; i < 3; ++i) {
@@ -2703,20 +3237,35 @@ bool encode_one(const KvView& kv, const StepParams& p, CUtensorMap* map, int* tp
 }  // namespace
 
 void encode_kv_maps(StepParams& p) {
+  const bool want_tc = p.use_tc != 0;
   p.use_tma = 0;
+  p.use_tc = 0;
   if (p.dtype != 0 || (p.D != 64 && p.D != 128)) return;
+  if (p.paged && p.page_size < 8) return;  // box origins must stay 1024-byte aligned in shared memory
+  const int R = p.paged ? (p.page_size < kTmaTile ? p.page_size : kTmaTile) : kTmaTile;
+  int kt = 0, kg = 0, kb = 0, vt = 0, vg = 0, vb = 0;
+  if (!encode_one(p.k, p, &p.tmk, &kt, &kg, &kb, R) || !encode_one(p.v, p, &p.tmv, &vt, &vg, &vb, R)) return;
+  if (kt != vt || kg != vg || kb != vb) return;  // both caches must share an axis order
+  p.tpos = kt; p.gpos = kg; p.bpos = kb;
+  if (want_tc && tc_eligible(p.dtype, p.D, p.G, p.paged, p.page_size)) {
+    // Page ids of a split's boxes are staged in shared memory: bound them
+    // (a split holds at most split_w + 1 tiles).
+    const int R2 = p.paged ? (p.page_size < kTcRows ? p.page_size : kTcRows) : kTcRows;
+    const int64_t boxes = p.paged ? (int64_t)(p.split_w + 1) * (kTcRows / R2) : 0;
+    if (boxes <= kTcMaxBoxes && encode_one(p.k, p, &p.tmk2, &kt, &kg, &kb, R2) &&
+        encode_one(p.v, p, &p.tmv2, &vt, &vg, &vb, R2) && kt == p.tpos && vt == p.tpos && kg == p.gpos &&
+        vg == p.gpos && kb == p.bpos && vb == p.bpos)
+      p.use_tc = 1;
+    p.use_tma = 1;
+    return;
+  }
   if (p.paged) {
-    if (p.page_size < 8) return;  // box origins must stay 1024-byte aligned in shared memory
     // Page ids of a CTA's boxes are staged in shared memory: bound them.
     const int64_t tiles = (p.max_seq + kTmaTile - 1) / kTmaTile;
     const int64_t per_cta = (2 * tiles + p.ns - 1) / p.ns + 1;
-    const int64_t boxes = per_cta * (kTmaTile / (p.page_size < kTmaTile ? p.page_size : kTmaTile));
+    const int64_t boxes = per_cta * (kTmaTile / R);
     if (boxes > kTmaMaxBoxes) return;
   }
-  int kt = 0, kg = 0, kb = 0, vt = 0, vg = 0, vb = 0;
-  if (!encode_one(p.k, p, &p.tmk, &kt, &kg, &kb) || !encode_one(p.v, p, &p.tmv, &vt, &vg, &vb)) return;
-  if (kt != vt || kg != vg || kb != vb) return;  // both caches must share an axis order
-  p.tpos = kt; p.gpos = kg; p.bpos = kb;
   p.use_tma = 1;
 }
 

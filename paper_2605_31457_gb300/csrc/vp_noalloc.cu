@@ -176,12 +176,10 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   p.mt_o = reinterpret_cast<float*>(base + L.o_mo);
   p.mt_st = reinterpret_cast<float*>(base + L.o_ms);
   p.hmax = reinterpret_cast<float*>(base + L.o_hm);
-  const vp::Plan pl = vp::make_plan(batch, Hkv, D, slot->num_sms, c.max_visual, c.max_seq, kept_cap,
-                                    budget->granularity);
   p.hp = L.hp;
-  p.ns = pl.ns; p.nsp_max = L.nsp_max; p.cl = pl.cl;
-  p.nk = pl.nk; p.nk_max = L.nk_max; p.nm = pl.nm; p.nc = pl.nc; p.gslice = pl.gslice; p.split_w = pl.split_w;
-  vp::encode_kv_maps(p);
+  p.nsp_max = L.nsp_max;
+  p.nk_max = L.nk_max;
+  vp::plan_step(p, slot->num_sms, kept_cap, budget->granularity);
   e = vp::launch_score(p, stream);
   if (e == cudaSuccess) e = vp::launch_select(p, stream);
   if (e == cudaSuccess) e = vp::launch_gather(p, stream);

@@ -35,6 +35,10 @@ VP_FIXED_K = 2
 VP_DENSE = 3
 VP_TOP_P = 4
 
+VP_SCORE_AUTO = 0
+VP_SCORE_MMA = 1
+VP_SCORE_TC = 2
+
 EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
             "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc")
 VP_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -77,6 +81,8 @@ lib.vp_decode_gather.argtypes = [_P, ctypes.c_int32, _P, ctypes.POINTER(vp_kv), 
 lib.vp_decode_gather.restype = ctypes.c_int
 lib.vp_set_diagnostics.argtypes = [_P, ctypes.c_float, _P, _P]
 lib.vp_set_diagnostics.restype = ctypes.c_int
+lib.vp_set_score_path.argtypes = [_P, ctypes.c_int32]
+lib.vp_set_score_path.restype = ctypes.c_int
 lib.vp_max_kept.argtypes = [ctypes.POINTER(vp_budget), ctypes.c_int32]
 lib.vp_max_kept.restype = ctypes.c_int32
 lib.vp_last_error.argtypes = [_P]
@@ -151,6 +157,12 @@ def vp_decode_gather(ctx, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span:
                               ctypes.byref(visual_span), _ptr(text_len), _ptr(kept_idx), int(kept_cap),
                               _ptr(kept_count), int(granularity), float(scale), _ptr(out), ctypes.c_void_p(stream))
     return _check(st, ctx) if check else st
+
+
+def vp_set_score_path(ctx, path):
+    """Score kernel of later vp_decode_step calls: VP_SCORE_AUTO, VP_SCORE_MMA
+    or VP_SCORE_TC."""
+    return _check(lib.vp_set_score_path(ctx, int(path)), ctx)
 
 
 def vp_set_diagnostics(ctx, delta, n_act=None, active_bits=None):

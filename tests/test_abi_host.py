@@ -60,6 +60,7 @@ def test_null_context_and_null_free(lib):
     assert lib.lib.vp_check_errors(None, None) == lib.VP_ERR_NOT_INITIALIZED
     st = lib.lib.vp_decode_gather(None, 1, None, None, None, None, None, None, 0, None, 0, 0.0, None, None)
     assert st == lib.VP_ERR_NOT_INITIALIZED
+    assert lib.lib.vp_set_score_path(None, lib.VP_SCORE_TC) == lib.VP_ERR_NOT_INITIALIZED
     lib.vp_free(None)
 
 

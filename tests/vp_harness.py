@@ -80,7 +80,8 @@ def place(x: torch.Tensor, layout: str, dev) -> torch.Tensor:
 class Device:
     """Device copies of an Inputs plus a library context and output buffers."""
 
-    def __init__(self, vp, inp: Inputs, budget: dict, max_batch=None, max_seq=None, layout="bhtd"):
+    def __init__(self, vp, inp: Inputs, budget: dict, max_batch=None, max_seq=None, layout="bhtd",
+                 score_path=None):
         self.vp = vp
         r = inp.recipe
         dev = torch.device("cuda")
@@ -92,6 +93,8 @@ class Device:
         self.cfg = vp.make_config(max_batch or r.batch, r.heads, r.kv_heads, r.head_dim, max_visual,
                                   max(max_seq, max_visual + 1), dtype, int(r.paged), r.page_size)
         self.ctx = vp.vp_init(self.cfg)
+        if score_path is not None:
+            vp.vp_set_score_path(self.ctx, score_path)
         self.q = inp.q.to(dev)
         if r.paged:
             pk = W.scatter_pages(inp.k, inp.block_table, inp.n_pages, r.page_size)
@@ -227,8 +230,8 @@ def compare_seq(inp: Inputs, gpu: dict, b: int, budget: dict, report: dict | Non
     return ref
 
 
-def check_all(vp, inp: Inputs, budget: dict, seqs=None, report=None, layout="bhtd"):
-    dev = Device(vp, inp, budget, layout=layout)
+def check_all(vp, inp: Inputs, budget: dict, seqs=None, report=None, layout="bhtd", score_path=None):
+    dev = Device(vp, inp, budget, layout=layout, score_path=score_path)
     try:
         gpu = dev.run()
     finally:
