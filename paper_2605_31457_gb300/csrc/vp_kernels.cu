@@ -1236,10 +1236,10 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 }
 // Barrier of the four softmax warps (named barrier 1); the second form also
 // counts the threads whose predicate is true.
-__device__ __forceinline__ void wg_sync() { asm volatile("bar.sync 1, 128;\n" ::: "memory"); }
+__device__ __forceinline__ void wg_sync() { asm volatile("barrier.cta.sync 1, 128;\n" ::: "memory"); }
 __device__ __forceinline__ int wg_sync_count(bool pred) {
   int n;
-  asm volatile("{\n .reg .pred p;\n setp.ne.b32 p, %1, 0;\n bar.red.popc.u32 %0, 1, 128, p;\n}\n"
+  asm volatile("{\n .reg .pred p;\n setp.ne.b32 p, %1, 0;\n barrier.cta.red.popc.u32 %0, 1, 128, p;\n}\n"
                : "=r"(n) : "r"((int)pred) : "memory");
   return n;
 }
@@ -1499,7 +1499,7 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
     for (int i = 0; i < n; ++i) {
       const int u = tr.u0 + i, sb = i & 1;
       float sv[16];
-      if (!dead && mbar_wait(s_full + sb, (i >> 1) & 1)) {
+      if (__all_sync(0xffffffffu, !dead && mbar_wait(s_full + sb, (i >> 1) & 1))) {
         tc_fence_after();
         tmem_ld16(taddr + 16 * sb, sv);
       } else {
@@ -1563,9 +1563,9 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
           mref[h] = mn;
         }
         wg_sync();  // red is read before its next use
-        if (j > 0 && !dead) {
+        if (j > 0 && __any_sync(0xffffffffu, !dead)) {
           // O holds the products of text tiles 0 .. j - 1: rescale it once the last is complete.
-          if (mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1)) {
+          if (__all_sync(0xffffffffu, !dead && mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1))) {
             tc_fence_after();
             float o[16];
             tmem_ld16(taddr + 32, o);
@@ -1604,8 +1604,8 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
     float o[16];
 #pragma unroll
     for (int h = 0; h < 16; ++h) o[h] = 0.f;
-    if (j > 0 && !dead) {
-      if (mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1)) {
+    if (j > 0 && __any_sync(0xffffffffu, !dead)) {
+      if (__all_sync(0xffffffffu, !dead && mbar_wait(pv_done + ((j - 1) & 1), ((j - 1) >> 1) & 1))) {
         tc_fence_after();
         tmem_ld16(taddr + 32, o);
       } else {
