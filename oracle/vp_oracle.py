@@ -22,6 +22,8 @@ one decode step t (VisionPulse, Sec. 4.2-4.3 and Sec. 5.2):
      the anchor's kept set, with no selection of its own         (Sec. 4.2, Sec. 5.1)
   9. the active visual token count N_act(delta) and the per-token
      activity flags behind persistent inactivity                   (Sec. 4.3, App. B)
+ 10. FastV prefill pruning before VisionPulse: the surviving visual tokens
+     and the cache that holds only them                              (App., prefill pruning)
 
 Everything is float64 computed from the exact input values (bf16 or fp32
 inputs are widened without rounding).  There is no blocking, fusion or
@@ -320,3 +322,40 @@ def active_count(s: np.ndarray, delta: float):
     """
     active = np.asarray(s, dtype=np.float32) > np.float32(delta)
     return active.sum(axis=-1), active
+
+
+def fastv_survivors(q_last, k, vis_start: int, vis_len: int, text_len: int, ratio_ppm: int = 500_000, *,
+                    scale: float = 0.0) -> np.ndarray:
+    """FastV's prefill-stage selection (the appendix "Complementarity with
+    Prefill Pruning": compression ratio 0.5, then VisionPulse decodes over
+    the rest).  FastV ranks visual tokens by the attention they receive from
+    the last prompt token at the pruning layer, averaged over heads -- the S
+    of Eq. 2 with that token as the query (Sec. 4.2 follows FastV's estimator
+    at every step) -- and keeps the top ratio, at least one token.
+
+    q_last: [H, D] query of the last prompt token; k: [Hkv, T, D].
+    Returns the kept visual indices, ascending, relative to vis_start.
+    """
+    q_last = np.asarray(q_last, dtype=np.float64)
+    H, D = q_last.shape
+    T = vis_len + text_len
+    if scale == 0.0:
+        scale = 1.0 / math.sqrt(D)
+    z = logits(q_last, np.asarray(k[:, :T], dtype=np.float64), scale)
+    vis = np.zeros(T, dtype=bool)
+    vis[vis_start:vis_start + vis_len] = True
+    s = importance(softmax_tau(z, 1.0), vis)
+    n_keep = budget(0.0, vis_len, mode=FIXED_RATIO, ratio_ppm=ratio_ppm)
+    return select_topk(s, n_keep)
+
+
+def compact_cache(x, vis_start: int, vis_len: int, text_len: int, kept) -> np.ndarray:
+    """The cache of one sequence after prefill pruning: the rows before the
+    visual span, the surviving visual rows in ascending order, then the rows
+    after the span.  x: [Hkv, T, D] with T >= vis_len + text_len.
+    Returns [Hkv, len(kept) + text_len, D]."""
+    x = np.asarray(x)
+    kept = np.asarray(kept, dtype=np.int64)
+    T = vis_len + text_len
+    rows = np.concatenate([np.arange(vis_start), vis_start + kept, np.arange(vis_start + vis_len, T)])
+    return x[:, rows]

@@ -450,3 +450,66 @@ def test_top_p_limits_and_monotonicity():
     dominant = np.r_[np.full(9, 0.02), 0.5]               # one token holds 0.5 / 0.68 = 74% of the scores
     assert O.top_p_budget(dominant, 100_000) == 1 and O.top_p_budget(dominant, 730_000) == 1
     assert O.top_p_budget(dominant, 750_000) == 2
+
+
+# ------------------------------------------------ FastV prefill pruning (appendix)
+
+def test_fastv_zero_query_keeps_the_first_half():
+    """q = 0: every visual token gets the same attention, so the tie rule keeps
+    the lowest indices; ratio 0.5 keeps ceil(N_v / 2), at least one."""
+    q, k, v, vs, nv, tl = _rand_case(80, n_v=13, text=4, vis_start=2)
+    assert list(O.fastv_survivors(np.zeros_like(q), k, vs, nv, tl)) == list(range(7))
+    assert list(O.fastv_survivors(np.zeros_like(q), k, vs, 1, tl)) == [0]
+
+
+def test_fastv_brute_force_and_planted_recall():
+    """Against explicit per-head loops on tiny inputs, and planted keys aligned
+    with the last prompt token's query are always among the survivors."""
+    for seed in range(5):
+        q, k, v, vs, nv, tl = _rand_case(81 + seed, H=4, Hkv=2, D=8, n_v=10, text=5, vis_start=3)
+        H, D = q.shape
+        G = H // k.shape[0]
+        T = nv + tl
+        s = np.zeros(nv)
+        for h in range(H):
+            z = [float(np.dot(q[h], k[h // G, j])) / math.sqrt(D) for j in range(T)]
+            m = max(z)
+            den = sum(math.exp(x - m) for x in z)
+            for i in range(nv):
+                s[i] += math.exp(z[vs + i] - m) / den / H
+        order = sorted(range(nv), key=lambda i: (-float(np.float32(s[i])), i))
+        assert list(O.fastv_survivors(q, k, vs, nv, tl)) == sorted(order[:5])
+    q, k, v, vs, nv, tl = _rand_case(90, H=4, Hkv=2, D=16, n_v=40, text=6)
+    for i in (3, 17, 31):
+        for g in range(2):
+            k[g, vs + i] = 4.0 * q[2 * g:2 * g + 2].mean(0) / np.linalg.norm(q[2 * g:2 * g + 2].mean(0)) * math.sqrt(16)
+    assert {3, 17, 31} <= set(O.fastv_survivors(q, k, vs, nv, tl, ratio_ppm=100_000).tolist())
+
+
+def test_compact_cache_rows():
+    """Rows labelled with their own position map as the definition says; with
+    every visual token kept the cache is unchanged."""
+    Hkv, T, D = 2, 30, 4
+    x = np.broadcast_to(np.arange(T, dtype=np.float64)[None, :, None], (Hkv, T, D)).copy()
+    vs, nv, tl = 4, 15, 15
+    kept = np.array([0, 2, 3, 9, 14])
+    c = O.compact_cache(x, vs, nv, tl, kept)
+    want = list(range(4)) + [4, 6, 7, 13, 18] + list(range(19, 30))
+    assert c.shape == (Hkv, len(kept) + tl, D)
+    assert c[0, :, 0].tolist() == want and c[1, :, 3].tolist() == want
+    assert np.array_equal(O.compact_cache(x, vs, nv, tl, np.arange(nv)), x)
+
+
+def test_compacted_decode_equals_attention_restricted_to_survivors():
+    """Dense attention over the compacted cache is the attention of the full
+    cache with the pruned visual tokens removed from the softmax set (the
+    anchor-layer attention with the survivors as its kept set), and a
+    VisionPulse step over the compacted cache keeps a subset of survivors."""
+    q, k, v, vs, nv, tl = _rand_case(91, H=4, Hkv=2, D=8, n_v=16, text=6, vis_start=2)
+    surv = O.fastv_survivors(q * 0.7, k, vs, nv, tl)
+    kc, vc = O.compact_cache(k, vs, nv, tl, surv), O.compact_cache(v, vs, nv, tl, surv)
+    dense = O.decode_step(q, kc, vc, vs, len(surv), tl, mode=O.DENSE)
+    want = O.anchor_attention(q, k, v, vs, nv, tl, [surv])
+    np.testing.assert_allclose(dense["out"], want, rtol=0, atol=1e-12)
+    r = O.decode_step(q, kc, vc, vs, len(surv), tl, mode=O.FIXED_RATIO, ratio_ppm=250_000)
+    assert set(surv[r["kept"][0]].tolist()) <= set(surv.tolist()) and len(r["kept"][0]) == 2
