@@ -45,7 +45,8 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=None, help="timed steps (default: the workload's)")
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--workload", default="qwen7b",
-                    help="qwen7b (default) | qwen7b-anchor | serving | long | sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
+                    help="qwen7b (default) | qwen7b-anchor | qwen7b-fastv-vp | serving | long | "
+                         "sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle CPU-baseline leg")
@@ -254,7 +255,7 @@ def workload_config(r, nbuf=None):
 def pick_workload(name):
     """(recipe, default timed steps, distinct layer caches, host-generated)."""
     from paper_2605_31457_gb300 import workloads as W
-    if name in ("qwen7b", "qwen7b-anchor"):
+    if name in ("qwen7b", "qwen7b-anchor", "qwen7b-fastv-vp"):
         return W.QWEN7B, 256, W.QWEN7B.layers, True
     if name == "serving":
         return W.SERVING, 64, 4, False
@@ -341,22 +342,64 @@ def run_ours(args, rank, world, local):
     # (Sec. 5.1, l_a = 17): layers 1-16 attend densely (the whole visual span
     # kept), layer 17 runs the VisionPulse step, layers 18-28 reuse its kept
     # set.  Every other workload treats each layer as its own anchor.
-    anchor = ANCHOR_LAYER if args.workload.endswith("-anchor") else None
+    anchor = ANCHOR_LAYER if args.workload.endswith(("-anchor", "-fastv-vp")) else None
     if anchor is not None:
         kept_all = torch.arange(nv_max, dtype=torch.int32, device=dev)[None, :].repeat(B, 1).contiguous()
         count_all = vis_len.clone()
+    # qwen7b-fastv-vp: FastV at the prefill stage (the paper's appendix on
+    # prefill pruning: ratio 0.5 at the pruning layer, ranked by the last
+    # prompt token's head-averaged attention -- Eq. 2 with that query), then
+    # the anchor pipeline over the survivors: layers from the anchor on read
+    # caches compacted to the surviving visual tokens.  The prefill stage runs
+    # once, before the timed decode, and is timed on its own.
+    fastv = args.workload.endswith("-fastv-vp")
+    kc_run, vc_run, span_run = list(kc), list(vc), [span] * L
+    prefill_ms = None
+    if fastv:
+        fv_budget = vp.make_budget(mode=vp.VP_FIXED_RATIO, tau=0.1, ratio_ppm=500_000)
+        fv_cap = max(1, vp.vp_max_kept(fv_budget, nv_max))
+        fv_kept = torch.empty((B, fv_cap), dtype=torch.int32, device=dev)
+        fv_count = torch.empty((B,), dtype=torch.int32, device=dev)
+        fv_out = torch.empty((B, H, D), dtype=cdt, device=dev)
+        fv_mass = torch.empty((B, H), dtype=torch.float32, device=dev)
+        tl_all = tl_steps[S - 1]  # every row a decode step will read, appended tokens included
+        comp = []
+        for layer in range(anchor, L):
+            shape = (B, Hkv, t_cap, D)
+            comp.append((torch.zeros(shape, dtype=cdt, device=dev), torch.zeros(shape, dtype=cdt, device=dev)))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        # The last prompt token's query at the pruning layer: the recipe's
+        # query for that layer (step 0), before any decode token.
+        vp.vp_decode_step(ctx, B, q_dev[0, anchor], kc[anchor % nbuf], vc[anchor % nbuf], span, tl_steps[0],
+                          fv_budget, fv_out, fv_kept, fv_cap, fv_count, fv_mass)
+        for i, layer in enumerate(range(anchor, L)):
+            for src, dst in ((kc[layer % nbuf], comp[i][0]), (vc[layer % nbuf], comp[i][1])):
+                vp.vp_compact_kv(ctx, B, src, vp.kv_contiguous(dst), span, tl_all, fv_kept, fv_cap, fv_count)
+        e1.record()
+        torch.cuda.synchronize()
+        prefill_ms = e0.elapsed_time(e1)
+        vp.vp_check_errors(ctx)
+        span_c = vp.span(vis_start, fv_count)
+        for i, layer in enumerate(range(anchor, L)):
+            kc_run[layer], vc_run[layer] = vp.kv_contiguous(comp[i][0]), vp.kv_contiguous(comp[i][1])
+            span_run[layer] = span_c
+        nvs_surv = fv_count.cpu().numpy().astype(np.int64)
 
     def step_calls(s, stream=None):
         for layer in range(L):
-            kcl, vcl = kc[layer % nbuf], vc[layer % nbuf]
+            kcl = kc_run[layer] if fastv else kc[layer % nbuf]
+            vcl = vc_run[layer] if fastv else vc[layer % nbuf]
+            spl = span_run[layer]
             if anchor is not None and layer < anchor:
-                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], kept_all, nv_max,
+                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, spl, tl_steps[s], kept_all, nv_max,
                                     count_all, out[layer], stream=stream)
             elif anchor is not None and layer > anchor:
-                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], kept[anchor], cap,
+                vp.vp_decode_gather(ctx, B, q_dev[s, layer], kcl, vcl, spl, tl_steps[s], kept[anchor], cap,
                                     count[s, anchor], out[layer], stream=stream)
             else:
-                vp.vp_decode_step(ctx, B, q_dev[s, layer], kcl, vcl, span, tl_steps[s], budget,
+                vp.vp_decode_step(ctx, B, q_dev[s, layer], kcl, vcl, spl, tl_steps[s], budget,
                                   out[layer], kept[layer], cap, count[s, layer], mass[layer], stats[s, layer],
                                   stream=stream)
 
@@ -421,7 +464,8 @@ def run_ours(args, rank, world, local):
         for layer in range(L):
             for b in range(B):
                 if anchor is None or layer == anchor:
-                    a, c = call_bytes(r, int(nvs[b]), int(tls[b]) + s, int(counts[s, layer, b]))
+                    nv_read = int(nvs_surv[b]) if fastv else int(nvs[b])  # the anchor's visual span
+                    a, c = call_bytes(r, nv_read, int(tls[b]) + s, int(counts[s, layer, b]))
                     score_bytes += a
                     gather_bytes += c
                 else:  # the visual rows read: all of them before the anchor, the kept ones after
@@ -464,10 +508,18 @@ def run_ours(args, rank, world, local):
         "gpu_launches": 3 * n_calls + (0 if anchor is None else 2 * args.steps * (L - 1)),
         "clocks": clocks,
     }
+    if fastv:
+        line["prefill_prune"] = {
+            "ms": prefill_ms, "visual_kept_frac": float(nvs_surv.sum() / nvs.sum()),
+            "note": (f"once before decoding: FastV selection at layer {anchor + 1} (vp_decode_step, fixed ratio 50%, "
+                     f"last prompt token's query) and vp_compact_kv of the K and V caches of layers "
+                     f"{anchor + 1}-{L}; not in the timed region")}
     if anchor is not None:
         line["config"]["pipeline"] = (f"anchor layer {anchor + 1} of {L}: layers 1-{anchor} dense attention "
                                       f"(vp_decode_gather, whole visual span kept), layer {anchor + 1} "
-                                      f"vp_decode_step, layers {anchor + 2}-{L} vp_decode_gather on its kept set")
+                                      f"vp_decode_step, layers {anchor + 2}-{L} vp_decode_gather on its kept set"
+                                      + (f"; layers {anchor + 1}-{L} read caches holding only FastV's prefill "
+                                         f"survivors (50% of the visual tokens)" if fastv else ""))
         line["roofline"]["timing"] += "; only the anchor layer's call is timed per kernel"
         line["hbm"]["note"] = ("whole step: algorithmic bytes (dense layers: all K/V; anchor layer: all visual K + "
                                "kept visual V + text K/V; later layers: kept visual K/V + text K/V; q + out) / step time")

@@ -200,6 +200,40 @@ vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
  */
 vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t* active_bits);
 
+/*
+ * Prefill-stage compaction for FastV + VisionPulse (the paper's appendix
+ * "Complementarity with Prefill Pruning": FastV prunes the visual tokens at
+ * the prefill stage with compression ratio 0.5, then VisionPulse prunes step
+ * by step over the remaining ones).  FastV ranks the visual tokens by the
+ * head-averaged attention of the last prompt token at the pruning layer
+ * (Sec. 5.1, l_a = 17) -- Eq. 2 with that token as the query -- so the
+ * selection is a vp_decode_step call with VP_FIXED_RATIO (ratio_ppm =
+ * 500000) and granularity 0 on that token; this call then writes, for one
+ * layer, a cache holding only the surviving visual tokens:
+ *   dst row t  =  src row t                      for t <  vis_start
+ *              =  src row vis_start + kept[t - vis_start]
+ *                                                 for vis_start <= t < vis_start + K
+ *              =  src row t - K + vis_len        for t >= vis_start + K, t < K + text_len
+ * with K = kept_count[b].  The compacted sequence has visual span
+ * (vis_start, K) -- kept_count itself can serve as the new vis_len array --
+ * and the same text_len.
+ *   src          a cache as for vp_decode_step (contiguous or paged, cfg.dtype).
+ *   dst          contiguous cache of cfg.dtype, caller-owned, rows for at
+ *                least max(K + text_len) tokens per (sequence, kv-head);
+ *                must not overlap src.
+ *   kept_idx     int32 [batch][kept_cap]: surviving visual indices (relative to
+ *                vis_start), ascending as vp_decode_step writes them.
+ *   kept_count   int32 [batch]; 0 <= kept_count <= min(kept_cap, vis_len).
+ * Asynchronous on cuda_stream; uses no workspace.  Out-of-range kept indices
+ * and unmapped pages are skipped (the row is zeroed) and flagged in the
+ * device error word (vp_check_errors).  Host-visible argument errors return
+ * VP_ERR_INVALID_ARG before anything is enqueued.
+ */
+vp_status vp_compact_kv(vp_ctx* ctx, int32_t batch, const vp_kv* src, const vp_kv* dst,
+                        const vp_span* visual_span, const int32_t* text_len,
+                        const int32_t* kept_idx, int32_t kept_cap, const int32_t* kept_count,
+                        void* cuda_stream);
+
 /* Score kernel of later vp_decode_step calls on this context (an
  * implementation choice with no counterpart in the paper; results agree
  * within the documented tolerances either way):

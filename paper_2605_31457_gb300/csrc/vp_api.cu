@@ -389,6 +389,48 @@ vp_status vp_set_diagnostics(vp_ctx* ctx, float delta, int32_t* n_act, uint32_t*
   return VP_OK;
 }
 
+vp_status vp_compact_kv(vp_ctx* ctx, int32_t batch, const vp_kv* src, const vp_kv* dst,
+                        const vp_span* visual_span, const int32_t* text_len,
+                        const int32_t* kept_idx, int32_t kept_cap, const int32_t* kept_count,
+                        void* cuda_stream) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  ctx->last_error.clear();
+  const vp_config& c = ctx->cfg;
+  if (batch < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: batch < 0");
+  if (batch > c.max_batch) return fail(ctx, VP_ERR_CAPACITY, "vp_compact_kv: batch exceeds max_batch");
+  if (kept_cap < 0) return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: kept_cap < 0");
+  if (batch == 0) return VP_OK;
+  if (!text_len || !visual_span || !visual_span->vis_start || !visual_span->vis_len || !kept_count ||
+      (kept_cap > 0 && !kept_idx))
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: NULL tensor argument");
+  std::string why;
+  if (!kv_ok(ctx, src, "src", &why)) return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: " + why);
+  const size_t esz = c.dtype == VP_BF16 ? 2 : 4;
+  if (!dst || !dst->data || !aligned16(dst->data) || dst->block_table)
+    return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: dst must be a contiguous cache with 16-byte-aligned data");
+  for (int64_t st : {dst->stride_b, dst->stride_h, dst->stride_t})
+    if (st < 0 || ((uint64_t)st * esz) % 16 != 0)
+      return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: dst strides must be >= 0 and multiples of 16 bytes");
+  if (dst->data == src->data) return fail(ctx, VP_ERR_INVALID_ARG, "vp_compact_kv: dst must not overlap src");
+  vp::CompactParams p;
+  memset(&p, 0, sizeof p);
+  p.src = vp::KvView{src->data, src->stride_b, src->stride_h, src->stride_t, src->block_table, src->max_pages,
+                     src->num_pages};
+  p.paged = c.paged;
+  p.page_size = c.paged ? c.page_size : 1;
+  while ((1 << p.page_shift) < p.page_size) ++p.page_shift;
+  p.dst = const_cast<void*>(dst->data);  // the destination cache is written
+  p.dsb = dst->stride_b; p.dsh = dst->stride_h; p.dst_t = dst->stride_t;
+  p.vis_start = visual_span->vis_start; p.vis_len = visual_span->vis_len; p.text_len = text_len;
+  p.kept_idx = kept_idx; p.kept_cap = kept_cap; p.kept_count = kept_count;
+  p.B = batch; p.Hkv = c.num_kv_heads; p.D = c.head_dim; p.esz = (int)esz;
+  p.max_visual = c.max_visual; p.max_seq = c.max_seq;
+  p.err = ctx->err;
+  const cudaError_t e = vp::launch_compact(p, static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return cuda_fail(ctx, "vp_compact_kv: launch", e);
+  return VP_OK;
+}
+
 vp_status vp_set_score_path(vp_ctx* ctx, int32_t path) {
   if (!ctx) return VP_ERR_NOT_INITIALIZED;
   ctx->last_error.clear();

@@ -201,6 +201,23 @@ inline WsLayout ws_layout(int batch, int H, int Hkv, int D, int max_visual, int 
   return w;
 }
 
+// Cache compaction for FastV + VisionPulse (vp_compact_kv).
+struct CompactParams {
+  KvView src;                  // contiguous or paged (block_table set)
+  int paged, page_size, page_shift;
+  void* dst;                   // contiguous destination
+  int64_t dsb, dsh, dst_t;     // its strides in elements
+  const int32_t* vis_start;
+  const int32_t* vis_len;
+  const int32_t* text_len;
+  const int32_t* kept_idx;
+  int kept_cap;
+  const int32_t* kept_count;
+  int B, Hkv, D, esz, max_visual, max_seq;
+  unsigned* err;
+};
+cudaError_t launch_compact(const CompactParams& c, cudaStream_t s);
+
 // Launchers (vp_kernels.cu).  Return the launch error, if any.
 cudaError_t launch_score(const StepParams& p, cudaStream_t s);
 cudaError_t launch_select(const StepParams& p, cudaStream_t s);

@@ -1665,6 +1665,65 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
 }
 
 // ---------------------------------------------------------------------------
+// k_compact: grid (row chunks, Hkv, B), 256 threads.  Writes the compacted
+// cache of one (sequence, kv-head): the rows before the visual span, the kept
+// visual rows in their order, then the rows after the span (vp_compact_kv).
+// Each thread copies 16-byte pieces; a warp covers whole rows, so the reads
+// of consecutive kept rows and of the text rows are coalesced per row.
+// ---------------------------------------------------------------------------
+constexpr int kCompactRows = 128;  // destination rows per CTA
+
+__global__ void __launch_bounds__(256) k_compact(const __grid_constant__ CompactParams c) {
+  pdl_wait();  // kept_idx / kept_count may come from the previous kernel
+  pdl_trigger();
+  const int g = blockIdx.y, b = blockIdx.z;
+  int vs = __ldg(c.vis_start + b), nv = __ldg(c.vis_len + b), tl = __ldg(c.text_len + b);
+  unsigned e = 0;
+  if (nv < 0 || nv > c.max_visual) { e |= ERR_SPAN; nv = min(max(nv, 0), c.max_visual); }
+  if (tl < 1) { e |= ERR_TEXT; tl = 1; }
+  if (nv + tl > c.max_seq) { e |= ERR_LEN; tl = max(1, c.max_seq - nv); }
+  if (vs < 0 || vs > tl) { e |= ERR_SPAN; vs = min(max(vs, 0), tl); }
+  int K = __ldg(c.kept_count + b);
+  if (K < 0 || K > min(c.kept_cap, nv)) { e |= ERR_KEPT; K = max(0, min(K, min(c.kept_cap, nv))); }
+  const int Tn = K + tl;  // rows of the compacted sequence
+  const int ppr = c.D * c.esz / 16;  // 16-byte pieces per row
+  const int rpi = 256 / ppr;         // rows per pass of the CTA
+  const int r0 = blockIdx.x * kCompactRows, r1 = min(Tn, r0 + kCompactRows);
+  const char* src = static_cast<const char*>(c.src.data);
+  char* dst = static_cast<char*>(c.dst);
+  for (int t = r0 + threadIdx.x / ppr; t < r1; t += rpi) {
+    const int piece = threadIdx.x % ppr;
+    int pos;  // source row
+    if (t < vs) {
+      pos = t;
+    } else if (t < vs + K) {
+      const int i = __ldg(c.kept_idx + (int64_t)b * c.kept_cap + (t - vs));
+      pos = (i >= 0 && i < nv) ? vs + i : -1;
+      if (pos < 0) e |= ERR_KEPT;
+    } else {
+      pos = t - K + nv;
+    }
+    const char* row = nullptr;
+    if (pos >= 0) {
+      if (c.paged) {
+        const int lp = pos >> c.page_shift;
+        const int page = lp < c.src.max_pages ? __ldg(c.src.block_table + (int64_t)b * c.src.max_pages + lp) : -1;
+        if (page >= 0 && page < c.src.num_pages)
+          row = src + ((int64_t)page * c.src.sb + (int64_t)g * c.src.sh + (int64_t)(pos & (c.page_size - 1)) * c.src.st) * c.esz;
+        else
+          e |= ERR_PAGE;
+      } else {
+        row = src + ((int64_t)b * c.src.sb + (int64_t)g * c.src.sh + (int64_t)pos * c.src.st) * c.esz;
+      }
+    }
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (row) v = __ldg(reinterpret_cast<const uint4*>(row) + piece);
+    reinterpret_cast<uint4*>(dst + ((int64_t)b * c.dsb + (int64_t)g * c.dsh + (int64_t)t * c.dst_t) * c.esz)[piece] = v;
+  }
+  if (e) atomicOr(c.err, e);
+}
+
+// ---------------------------------------------------------------------------
 // k_score_f32 (fp32 caches): lane-per-token dot products on the FMA pipes,
 // lane-per-dimension P.V; the same partials as k_score_mma.
 // ---------------------------------------------------------------------------
@@ -3166,6 +3225,19 @@ cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
   if (p.dtype == 0)
     return p.D == 128 ? launch_gather_td<__nv_bfloat16, 128>(p, st) : launch_gather_td<__nv_bfloat16, 64>(p, st);
   return p.D == 128 ? launch_gather_td<float, 128>(p, st) : launch_gather_td<float, 64>(p, st);
+}
+
+cudaError_t launch_compact(const CompactParams& c, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((c.max_seq + kCompactRows - 1) / kCompactRows, c.Hkv, c.B);
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_compact, c);
 }
 
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {

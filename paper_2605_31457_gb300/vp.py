@@ -40,7 +40,8 @@ VP_SCORE_MMA = 1
 VP_SCORE_TC = 2
 
 EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
-            "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc")
+            "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc", "vp_decode_gather",
+            "vp_set_diagnostics", "vp_set_score_path", "vp_compact_kv")
 VP_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -81,6 +82,9 @@ lib.vp_decode_gather.argtypes = [_P, ctypes.c_int32, _P, ctypes.POINTER(vp_kv), 
 lib.vp_decode_gather.restype = ctypes.c_int
 lib.vp_set_diagnostics.argtypes = [_P, ctypes.c_float, _P, _P]
 lib.vp_set_diagnostics.restype = ctypes.c_int
+lib.vp_compact_kv.argtypes = [_P, ctypes.c_int32, ctypes.POINTER(vp_kv), ctypes.POINTER(vp_kv),
+                              ctypes.POINTER(vp_span), _P, _P, ctypes.c_int32, _P, _P]
+lib.vp_compact_kv.restype = ctypes.c_int
 lib.vp_set_score_path.argtypes = [_P, ctypes.c_int32]
 lib.vp_set_score_path.restype = ctypes.c_int
 lib.vp_max_kept.argtypes = [ctypes.POINTER(vp_budget), ctypes.c_int32]
@@ -156,6 +160,20 @@ def vp_decode_gather(ctx, batch, q, k_cache: vp_kv, v_cache: vp_kv, visual_span:
     st = lib.vp_decode_gather(ctx, int(batch), _ptr(q), ctypes.byref(k_cache), ctypes.byref(v_cache),
                               ctypes.byref(visual_span), _ptr(text_len), _ptr(kept_idx), int(kept_cap),
                               _ptr(kept_count), int(granularity), float(scale), _ptr(out), ctypes.c_void_p(stream))
+    return _check(st, ctx) if check else st
+
+
+def vp_compact_kv(ctx, batch, src: vp_kv, dst: vp_kv, visual_span: vp_span, text_len, kept_idx, kept_cap,
+                  kept_count, stream=None, check=True):
+    """Writes into ``dst`` (contiguous) the cache ``src`` with only the kept
+    visual rows (FastV prefill pruning followed by VisionPulse)."""
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream().cuda_stream
+    elif hasattr(stream, "cuda_stream"):
+        stream = stream.cuda_stream
+    st = lib.vp_compact_kv(ctx, int(batch), ctypes.byref(src), ctypes.byref(dst), ctypes.byref(visual_span),
+                           _ptr(text_len), _ptr(kept_idx), int(kept_cap), _ptr(kept_count), ctypes.c_void_p(stream))
     return _check(st, ctx) if check else st
 
 
