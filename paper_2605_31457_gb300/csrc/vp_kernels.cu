@@ -2618,7 +2618,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // ---------------------------------------------------------------------------
 constexpr int kGmWarps = 4;
 constexpr int kGmSlots = 3;
-constexpr int kGmMaxChunk = 1024;  // kept rows per CTA (the plan's chunks are at most this)
+constexpr int kGmMaxChunk = 2048;  // kept rows per CTA (the plan's chunks are at most this)
 
 template <int D, int NT>
 struct GmCfg {
