@@ -33,6 +33,8 @@
 #include <math_constants.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "vp_internal.h"
 
 namespace cg = cooperative_groups;
@@ -1993,7 +1995,13 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   const int hbeg = p.granularity ? gsel * p.G : 0;
   const int hcnt = p.granularity ? p.G : H;
   const bool vec = (hbeg & 3) == 0 && (hcnt & 3) == 0;
-  const bool pre = NTH <= 512 && vec && hcnt <= 32 && i0 + tid < i1;
+  // Long slices (the 1024-thread form, slices above kSelSliceSmall) take the
+  // row-shared importance loop below; short ones (the B = 1 decode) request
+  // each thread's first row now.  The 512-thread form is compiled without the
+  // row-shared loop: its launches are latency-bound, and the larger code
+  // measured slower there.
+  const bool wide = NTH >= 1024 && vec && hcnt >= 4 && hcnt <= 32 && (i1 - i0) > 2 * NTH;
+  const bool pre = !wide && NTH <= 512 && vec && hcnt <= 32 && i0 + tid < i1;
   float4 zpre[8];
   if (pre) {
     const float4* zr = reinterpret_cast<const float4*>(p.z_ws + ((int64_t)b * p.max_visual + i0 + tid) * p.hp + hbeg);
@@ -2078,33 +2086,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   const bool diag = p.n_act || p.act_bits;
   int n_on = 0;
   float vsum = 0.f;  // top-p: this thread's share of the visual score total
-  for (int i = i0 + tid; i < i1; i += NTH) {
-    const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
-    float a = 0.f;
-    if (pre && i == i0 + tid) {
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        if (4 * q < hcnt) {
-          const int h = hbeg + 4 * q;
-          a = fmaf(fexp2_rel(zpre[q].x, hM_s[h]), hInv_s[h], a);
-          a = fmaf(fexp2_rel(zpre[q].y, hM_s[h + 1]), hInv_s[h + 1], a);
-          a = fmaf(fexp2_rel(zpre[q].z, hM_s[h + 2]), hInv_s[h + 2], a);
-          a = fmaf(fexp2_rel(zpre[q].w, hM_s[h + 3]), hInv_s[h + 3], a);
-        }
-      }
-    } else if (vec) {
-      for (int hh = 0; hh < hcnt; hh += 4) {
-        const float4 z4 = __ldcg(reinterpret_cast<const float4*>(zr + hh));
-        const int h = hbeg + hh;
-        a = fmaf(fexp2_rel(z4.x, hM_s[h]), hInv_s[h], a);
-        a = fmaf(fexp2_rel(z4.y, hM_s[h + 1]), hInv_s[h + 1], a);
-        a = fmaf(fexp2_rel(z4.z, hM_s[h + 2]), hInv_s[h + 2], a);
-        a = fmaf(fexp2_rel(z4.w, hM_s[h + 3]), hInv_s[h + 3], a);
-      }
-    } else {
-      for (int hh = 0; hh < hcnt; ++hh)
-        a = fmaf(fexp2_rel(__ldcg(zr + hh), hM_s[hbeg + hh]), hInv_s[hbeg + hh], a);
-    }
+  auto emit = [&](int i, float a) {  // a: sum over the heads of exp2(z - M_h) / L_h
     const float sc = a * inv_cnt;
     if (!isfinite(sc)) bad = 1;
     key0[i] = __float_as_uint(sc);
@@ -2112,6 +2094,103 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     if (diag && __float_as_uint(sc) > p.act_delta_bits) {  // S_i > delta (Sec. 4.3)
       ++n_on;
       if (p.act_bits) atomicOr(p.act_bits + ((int64_t)b * nsel + gsel) * p.act_words + (i >> 5), 1u << (i & 31));
+    }
+  };
+  // Long slices: LPT lanes share a token row, each reading one float4 of its
+  // heads, so that a warp's load covers consecutive rows; eight loads per
+  // lane are in flight, and a reduce-scatter over the LPT lanes leaves every
+  // lane whole-token sums to emit.
+  auto wide_loop = [&](auto lpt_tag) {
+    constexpr int LPT = decltype(lpt_tag)::value, TPI = 32 / LPT, V = 8;
+    const int Q = hcnt / 4, lq = lane % LPT;
+    const bool qok = lq < Q;
+    float m4[4], i4[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int h = hbeg + 4 * lq + c;
+      m4[c] = qok ? hM_s[h] : 0.f;
+      i4[c] = qok ? hInv_s[h] : 0.f;
+    }
+    const float* zb = p.z_ws + (int64_t)b * p.max_visual * p.hp + hbeg + 4 * lq;
+    int off = 0;  // first of this lane's V / LPT values after the reduce-scatter
+#pragma unroll
+    for (int s_ = 0; s_ < 3; ++s_)
+      if ((LPT >> (s_ + 1)) > 0 && (lane & (LPT >> (s_ + 1)))) off += V >> (s_ + 1);
+    for (int base = i0 + warp * V * TPI; base < i1; base += NW * V * TPI) {
+      float4 zz[V];
+#pragma unroll
+      for (int j = 0; j < V; ++j) {
+        const int tok = base + j * TPI + lane / LPT;
+        zz[j] = (qok && tok < i1) ? __ldcg(reinterpret_cast<const float4*>(zb + (int64_t)tok * p.hp))
+                                  : make_float4(-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F);
+      }
+      float v[V];
+#pragma unroll
+      for (int j = 0; j < V; ++j) {
+        float a = fexp2_rel(zz[j].x, m4[0]) * i4[0];
+        a = fmaf(fexp2_rel(zz[j].y, m4[1]), i4[1], a);
+        a = fmaf(fexp2_rel(zz[j].z, m4[2]), i4[2], a);
+        v[j] = fmaf(fexp2_rel(zz[j].w, m4[3]), i4[3], a);
+      }
+#pragma unroll
+      for (int s_ = 0; s_ < 3; ++s_) {
+        const int o = LPT >> (s_ + 1), half = V >> (s_ + 1);
+        if (o == 0) break;
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int k = 0; k < half; ++k) {
+          const float send = up ? v[k] : v[k + half];
+          const float keep = up ? v[k + half] : v[k];
+          v[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < V / LPT; ++k) {
+        const int tok = base + (k + off) * TPI + lane / LPT;
+        if (tok < i1) emit(tok, v[k]);
+      }
+    }
+  };
+  bool done = false;
+  if constexpr (NTH >= 1024) {
+    if (wide) {
+      const int Q = hcnt / 4;
+      if (Q <= 1) wide_loop(std::integral_constant<int, 1>{});
+      else if (Q <= 2) wide_loop(std::integral_constant<int, 2>{});
+      else if (Q <= 4) wide_loop(std::integral_constant<int, 4>{});
+      else wide_loop(std::integral_constant<int, 8>{});
+      done = true;
+    }
+  }
+  if (!done) {
+    for (int i = i0 + tid; i < i1; i += NTH) {
+      const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
+      float a = 0.f;
+      if (pre && i == i0 + tid) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (4 * q < hcnt) {
+            const int h = hbeg + 4 * q;
+            a = fmaf(fexp2_rel(zpre[q].x, hM_s[h]), hInv_s[h], a);
+            a = fmaf(fexp2_rel(zpre[q].y, hM_s[h + 1]), hInv_s[h + 1], a);
+            a = fmaf(fexp2_rel(zpre[q].z, hM_s[h + 2]), hInv_s[h + 2], a);
+            a = fmaf(fexp2_rel(zpre[q].w, hM_s[h + 3]), hInv_s[h + 3], a);
+          }
+        }
+      } else if (vec) {
+        for (int hh = 0; hh < hcnt; hh += 4) {
+          const float4 z4 = __ldcg(reinterpret_cast<const float4*>(zr + hh));
+          const int h = hbeg + hh;
+          a = fmaf(fexp2_rel(z4.x, hM_s[h]), hInv_s[h], a);
+          a = fmaf(fexp2_rel(z4.y, hM_s[h + 1]), hInv_s[h + 1], a);
+          a = fmaf(fexp2_rel(z4.z, hM_s[h + 2]), hInv_s[h + 2], a);
+          a = fmaf(fexp2_rel(z4.w, hM_s[h + 3]), hInv_s[h + 3], a);
+        }
+      } else {
+        for (int hh = 0; hh < hcnt; ++hh)
+          a = fmaf(fexp2_rel(__ldcg(zr + hh), hM_s[hbeg + hh]), hInv_s[hbeg + hh], a);
+      }
+      emit(i, a);
     }
   }
   if (bad) atomicOr(p.err, ERR_NONFINITE);
