@@ -2327,6 +2327,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     if (K >= nv) krem = 0;
   }
   bool take_all = K >= nv;
+  bool whole = false;  // the radix select stopped at a bucket kept whole (no tie to split)
   if (!topp && K > 0 && !take_all) {
     uint32_t prefix = 0, mask = 0;
     krem = (unsigned)K;
@@ -2381,8 +2382,14 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
       prefix |= dsel << shift;
       mask |= 255u << shift;
       if (shift == 0) n_theta = cnt;
+      if (shift > 0 && krem == cnt) {  // the whole bucket is kept: the threshold is its lowest key
+        whole = true;
+        break;
+      }
     }
-    theta = prefix;  // the K-th largest key; krem keys equal to it are kept
+    // The K-th largest key (krem keys equal to it are kept), or, when a
+    // bucket is kept whole, every key from its lowest possible value up.
+    theta = whole ? prefix - 1u : prefix;
   }
 
   // 5. Ascending compaction: keys above theta, plus the first krem equal keys
@@ -2391,7 +2398,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     // An odd chunk length keeps the threads' reads in distinct banks.
     const int per_t = ((nv + NTH - 1) / NTH) | 1;
     const int j0 = min(nv, tid * per_t), j1 = min(nv, j0 + per_t);
-    const bool ties = !take_all && krem < n_theta;
+    const bool ties = !take_all && !whole && krem < n_theta;
     int n_eq = 0;
     if (ties)
       for (int i = j0; i < j1; ++i) n_eq += key_s[i] == theta;
@@ -2402,7 +2409,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
       int r = eq_before;
       for (int i = j0; i < j1; ++i) {
         const uint32_t k = key_s[i];
-        const bool sel = take_all || k > theta || (k == theta && (unsigned)r < krem);
+        const bool sel = take_all || k > theta || (!whole && k == theta && (unsigned)r < krem);
         r += k == theta;
         n_sel += sel;
       }
@@ -2411,7 +2418,7 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
     int r = eq_before;
     for (int i = j0; i < j1; ++i) {
       const uint32_t k = key_s[i];
-      const bool sel = take_all || k > theta || (k == theta && (unsigned)r < krem);
+      const bool sel = take_all || k > theta || (!whole && k == theta && (unsigned)r < krem);
       r += k == theta;
       if (sel && o < K) kept[o++] = i;
     }
