@@ -83,12 +83,20 @@ __device__ __forceinline__ float group_sum(float x) {
   return x + __shfl_xor_sync(0xffffffffu, x, 16);
 }
 
+// exp2 by the hardware approximation (ex2.approx: a few ulp, subnormal
+// results flushed to 0), one instruction: the statistics merges run it on
+// every split record, in kernels whose launches are latency-bound.
+__device__ __forceinline__ float ex2_hw(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 // exp2(a - m) with an empty term (a = -inf) giving exactly 0.
 __device__ __forceinline__ float exp2_rel(float a, float m) {
-  return a == -CUDART_INF_F ? 0.f : exp2f(a - m);
+  return a == -CUDART_INF_F ? 0.f : ex2_hw(a - m);
 }
 __device__ __forceinline__ float exp2_tau(float a, float m, float inv_tau) {
-  return a == -CUDART_INF_F ? 0.f : exp2f((a - m) * inv_tau);
+  return a == -CUDART_INF_F ? 0.f : ex2_hw((a - m) * inv_tau);
 }
 
 template <typename T> __device__ __forceinline__ T from_f(float x);
