@@ -19,6 +19,7 @@ from __future__ import annotations
 
 import argparse
 import ctypes
+import dataclasses
 import hashlib
 import json
 import math
@@ -45,7 +46,7 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=None, help="timed steps (default: the workload's)")
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--workload", default="qwen7b",
-                    help="qwen7b (default) | qwen7b-anchor | qwen7b-fastv-vp | serving | long | "
+                    help="qwen7b (default) | qwen7b-10pct | qwen7b-anchor | qwen7b-fastv-vp | serving | long | "
                          "sweep-<N_v>-<r1|r5|r20|r50|adaptive>")
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
@@ -257,6 +258,8 @@ def pick_workload(name):
     from paper_2605_31457_gb300 import workloads as W
     if name in ("qwen7b", "qwen7b-anchor", "qwen7b-fastv-vp"):
         return W.QWEN7B, 256, W.QWEN7B.layers, True
+    if name == "qwen7b-10pct":  # the paper's 10% setting: tau = 0.4, clamp [5%, 10%]
+        return dataclasses.replace(W.QWEN7B, budget=W.ADAPTIVE_10PCT), 256, W.QWEN7B.layers, True
     if name == "serving":
         return W.SERVING, 64, 4, False
     if name == "long":
