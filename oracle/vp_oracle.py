@@ -29,7 +29,7 @@ Everything is float64 computed from the exact input values (bf16 or fp32
 inputs are widened without rounding).  There is no blocking, fusion or
 reordering beyond the definitions above.
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
   * Eq. 2 uses the plain softmax (tau = 1); tau enters only the mass (Eq. 6).
   * H is the number of query heads; under grouped-query attention query head h
     reads kv-head h // G with G = H / Hkv.
