@@ -2702,9 +2702,11 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // k_gather_mma (bf16): grid (nc, Hkv, B), 4 warps.  CTA c (a) attends over
 // chunk c of the kept list (c < nk).  Warp w takes 32-token tiles w, w + 4,
 // ... of the chunk and streams the kept V rows through a private ring of
-// three slots: lane t bulk-copies row t of a tile into a row padded to
-// 2D + 16 bytes (conflict-free ldmatrix), after lane 0 armed the slot's
-// mbarrier with the tile's byte count.  The tile's logits (read one tile
+// S slots (three; one when no chunk holds more than a tile per warp, so that
+// the smaller shared-memory footprint lets four CTAs share an SM): lane t
+// bulk-copies row t of a tile into a row padded to 2D + 16 bytes
+// (conflict-free ldmatrix), after lane 0 armed the slot's mbarrier with the
+// tile's byte count.  The tile's logits (read one tile
 // ahead) give per-head running maxima and probabilities; P.V runs on the
 // tensor cores as in the score kernel (A = V^T by ldmatrix.trans, B = P^T
 // from a per-warp bf16 buffer).  The warps' partials are merged into the
@@ -2714,34 +2716,38 @@ constexpr int kGmWarps = 4;
 constexpr int kGmSlots = 3;
 constexpr int kGmMaxChunk = 2048;  // kept rows per CTA (the plan's chunks are at most this)
 
-template <int D, int NT>
+template <int D, int NT, int S>
 struct GmCfg {
   static constexpr int GM = 8 * NT;
   static constexpr int THREADS = 32 * kGmWarps;
   static constexpr int MT = D / 16;
   static constexpr int HALF_BYTES = 32 * 128;                   // 32 rows x 64 dimensions
   static constexpr int SLOT = (D / 64) * HALF_BYTES;            // 32 V rows, swizzled
-  static constexpr int RING = kGmWarps * kGmSlots * SLOT;
+  // Kept rows per CTA: a single slot serves one tile per warp.
+  static constexpr int MAX_CHUNK = S == 1 ? 32 * kGmWarps : kGmMaxChunk;
+  // After part (a) the ring holds the warps' outputs, then the split weights;
+  // before it, the split weights of part (b).
+  static constexpr int OFF_TW = kGmWarps * GM * D * 4;
+  static constexpr int RING_BYTES = kGmWarps * S * SLOT;
+  static constexpr int REUSE_BYTES = OFF_TW + 2 * GM * kNsMax * 4;
+  static constexpr int RING = RING_BYTES > REUSE_BYTES ? RING_BYTES : REUSE_BYTES;
   static constexpr int OFF_BAR = RING;                          // full[warps][slots]
   // Logits of a slot's tokens, float [GM][32]; once read, the tile's bf16
   // probabilities [GM][32] take their place.
-  static constexpr int OFF_Z = OFF_BAR + kGmWarps * kGmSlots * 8;
-  static constexpr int OFF_MASK = OFF_Z + kGmWarps * kGmSlots * GM * 32 * 4;   // copied rows per slot
-  static constexpr int OFF_WST = OFF_MASK + kGmWarps * kGmSlots * 4;          // float [warps][GM][2]
-  static constexpr int OFF_FIN = OFF_WST + kGmWarps * GM * 2 * 4;             // float [GM][4]
+  static constexpr int OFF_Z = OFF_BAR + kGmWarps * S * 8;
+  static constexpr int OFF_MASK = OFF_Z + kGmWarps * S * GM * 32 * 4;   // copied rows per slot
+  static constexpr int OFF_WST = OFF_MASK + kGmWarps * S * 4;           // float [warps][GM][2]
+  static constexpr int OFF_FIN = OFF_WST + kGmWarps * GM * 2 * 4;       // float [GM][4]
   static constexpr int OFF_LAST = OFF_FIN + GM * 4 * 4;
-  static constexpr int OFF_KIDX = OFF_LAST + 16;                // int16 [kGmMaxChunk] kept indices
-  static constexpr size_t SMEM = (size_t)OFF_KIDX + kGmMaxChunk * 2;
-  // After part (a) the ring holds the warps' outputs, then the split weights.
-  static constexpr int OFF_TW = kGmWarps * GM * D * 4;
-  static_assert(OFF_TW + 2 * GM * kNsMax * 4 <= RING, "reuse of the ring");
-  static_assert(OFF_Z % 16 == 0 && OFF_WST % 16 == 0, "alignment");
+  static constexpr int OFF_KIDX = OFF_LAST + 16;                // int16 [MAX_CHUNK] kept indices
+  static constexpr size_t SMEM = (size_t)OFF_KIDX + MAX_CHUNK * 2;
+  static_assert(OFF_BAR % 8 == 0 && OFF_Z % 16 == 0 && OFF_WST % 16 == 0, "alignment");
 };
 
-template <int D, int NT>
+template <int D, int NT, int S>
 __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_constant__ StepParams p) {
-  using C = GmCfg<D, NT>;
-  constexpr int GM = C::GM, S = kGmSlots;
+  using C = GmCfg<D, NT, S>;
+  constexpr int GM = C::GM;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char* smem = smem_raw;
   const int c = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
@@ -2790,8 +2796,8 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
     const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
     const int per = (K + p.nk - 1) / p.nk;
-    const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + kGmMaxChunk));
-    if (per > kGmMaxChunk) err |= ERR_KEPT;  // the plan keeps every chunk within the limit
+    const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + C::MAX_CHUNK));
+    if (per > C::MAX_CHUNK) err |= ERR_KEPT;  // the plan keeps every chunk within the limit
     // The chunk's kept indices, read once (out-of-range ones become -1).
     for (int j = j0 + tid; j < j1; j += C::THREADS) {
       int i = __ldg(kept + j);
@@ -3239,8 +3245,15 @@ cudaError_t launch_gather_td(const StepParams& p, cudaStream_t st) {
   }
   const dim3 grid(p.nc, p.Hkv, p.B);
   if (sizeof(T) == 2) {
-    if (p.G <= 8) return launch_ex(k_gather_mma<D, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 1>::SMEM, st, 1, p);
-    return launch_ex(k_gather_mma<D, 2>, grid, dim3(32 * kGmWarps), GmCfg<D, 2>::SMEM, st, 1, p);
+    // A single ring slot when no chunk can hold more than one tile per warp.
+    const int kmax = min(p.kept_cap, p.max_visual);
+    const bool one = p.nk == 0 || (kmax + p.nk - 1) / p.nk <= GmCfg<D, 1, 1>::MAX_CHUNK;
+    if (p.G <= 8) {
+      if (one) return launch_ex(k_gather_mma<D, 1, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 1, 1>::SMEM, st, 1, p);
+      return launch_ex(k_gather_mma<D, 1, kGmSlots>, grid, dim3(32 * kGmWarps), GmCfg<D, 1, kGmSlots>::SMEM, st, 1, p);
+    }
+    if (one) return launch_ex(k_gather_mma<D, 2, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 2, 1>::SMEM, st, 1, p);
+    return launch_ex(k_gather_mma<D, 2, kGmSlots>, grid, dim3(32 * kGmWarps), GmCfg<D, 2, kGmSlots>::SMEM, st, 1, p);
   }
   if (p.G <= 4) return launch_ex(k_gather<T, D, 4>, grid, dim3(kGatherThreads), gather_smem<T, D, 4>(), st, 1, p);
   if (p.G <= 8) return launch_ex(k_gather<T, D, 8>, grid, dim3(kGatherThreads), gather_smem<T, D, 8>(), st, 1, p);
@@ -3257,10 +3270,14 @@ cudaError_t configure_fixed_kernels() {
 #define VP_SET(kernel, bytes) if (e == cudaSuccess) e = set_smem(kernel, bytes)
   VP_SET((k_score_tc<8>), (TcCfg::SMEM));
   VP_SET((k_score_tc<16>), (TcCfg::SMEM));
-  VP_SET((k_gather_mma<128, 1>), (GmCfg<128, 1>::SMEM));
-  VP_SET((k_gather_mma<128, 2>), (GmCfg<128, 2>::SMEM));
-  VP_SET((k_gather_mma<64, 1>), (GmCfg<64, 1>::SMEM));
-  VP_SET((k_gather_mma<64, 2>), (GmCfg<64, 2>::SMEM));
+  VP_SET((k_gather_mma<128, 1, kGmSlots>), (GmCfg<128, 1, kGmSlots>::SMEM));
+  VP_SET((k_gather_mma<128, 2, kGmSlots>), (GmCfg<128, 2, kGmSlots>::SMEM));
+  VP_SET((k_gather_mma<64, 1, kGmSlots>), (GmCfg<64, 1, kGmSlots>::SMEM));
+  VP_SET((k_gather_mma<64, 2, kGmSlots>), (GmCfg<64, 2, kGmSlots>::SMEM));
+  VP_SET((k_gather_mma<128, 1, 1>), (GmCfg<128, 1, 1>::SMEM));
+  VP_SET((k_gather_mma<128, 2, 1>), (GmCfg<128, 2, 1>::SMEM));
+  VP_SET((k_gather_mma<64, 1, 1>), (GmCfg<64, 1, 1>::SMEM));
+  VP_SET((k_gather_mma<64, 2, 1>), (GmCfg<64, 2, 1>::SMEM));
   VP_SET((k_score_tma<128, 1, kTmaWarps, tma_slots<128>(), false>), (tma_smem<128, 1>()));
   VP_SET((k_score_tma<128, 2, kTmaWarps, tma_slots<128>(), false>), (tma_smem<128, 2>()));
   VP_SET((k_score_tma<64, 1, kTmaWarps, tma_slots<64>(), false>), (tma_smem<64, 1>()));

@@ -131,17 +131,24 @@ def _many(batch, **kw):
     return small(batch=batch, vis_len=vis, vis_start=start, text_len=text, **kw)
 
 
-@pytest.mark.parametrize("dtype,D,batch,budget", [
-    (W.FP32, 64, 3, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000)),
-    (W.FP32, 128, 3, dict(mode=O.DENSE, tau=0.1)),
-    (W.BF16, 128, 40, W.ADAPTIVE_5PCT),
-    (W.BF16, 64, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000)),
-    (W.BF16, 128, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000, granularity=1)),
+@pytest.mark.parametrize("dtype,D,batch,budget,heads", [
+    (W.FP32, 64, 3, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000), (28, 4)),
+    (W.FP32, 128, 3, dict(mode=O.DENSE, tau=0.1), (28, 4)),
+    (W.BF16, 128, 40, W.ADAPTIVE_5PCT, (28, 4)),
+    (W.BF16, 64, 40, W.ADAPTIVE_5PCT, (28, 4)),
+    (W.BF16, 128, 40, W.ADAPTIVE_5PCT, (32, 2)),
+    (W.BF16, 64, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000), (28, 4)),
+    (W.BF16, 128, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000, granularity=1), (28, 4)),
+    (W.BF16, 128, 40, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000), (32, 2)),
 ])
-def test_chunk_gather_paths(vp, dtype, D, batch, budget):
+def test_chunk_gather_paths(vp, dtype, D, batch, budget, heads):
     """Kept sets above 256 rows (fp32 and bf16 chunk kernels), and many
-    sequences with small kept sets, which also take the chunk kernel."""
-    r = _many(batch, dtype=dtype, head_dim=D) if batch > 3 else small(dtype=dtype, head_dim=D)
+    sequences with small kept sets, which also take the chunk kernel (with a
+    single ring slot when no chunk exceeds one 32-row tile per warp); up to
+    8 and 16 query heads per kv-head."""
+    H, Hkv = heads
+    kw = dict(dtype=dtype, head_dim=D, heads=H, kv_heads=Hkv)
+    r = _many(batch, **kw) if batch > 3 else small(**kw)
     Hn.check_all(vp, Hn.make_inputs(r), budget)
 
 
