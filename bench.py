@@ -492,6 +492,7 @@ def run_ours(args, rank, world, local):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "tokens_per_s": value * r.batch,
         "config": dict(workload_config(r, nbuf), parallelism=f"replicas x{world}" if world > 1 else "single GPU"),
         "hbm": {"achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
                 "frac_of_nominal_8tbs": step_gbs / NOMINAL_HBM_GBS,
