@@ -65,6 +65,24 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(x, world, device):
+    """The largest value of x over all ranks (x itself with one rank): every
+    replica's timed region is bracketed by barriers and the slowest one sets
+    the job's time."""
+    if world <= 1:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, steps, seconds):
+    """Whole-job steps/s of `world` replicas that each ran `steps` steps in
+    (at most) `seconds`."""
+    return world * steps / seconds
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -446,11 +464,8 @@ def run_ours(args, rank, world, local):
         ev1.record()
         torch.cuda.synchronize()
         clk = sampler.stop() if sampler else None
-        el = ev0.elapsed_time(ev1)
+        el = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
         if world > 1:
-            t = torch.tensor([el], dtype=torch.float64, device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            el = float(t.item())
             torch.distributed.barrier()
         return el, clk
 
@@ -483,7 +498,7 @@ def run_ours(args, rank, world, local):
     achieved = score_bytes / (score_ms * 1e-3) / 1e9
     traffic = committed_traffic()
     ms_per_step = elapsed_ms / args.steps
-    value = world * args.steps / (elapsed_ms * 1e-3)
+    value = job_rate(world, args.steps, elapsed_ms * 1e-3)
     step_gbs = (score_bytes + gather_bytes + other_bytes) / (elapsed_ms * 1e-3) / 1e9
     kept_layers = list(range(L)) if anchor is None else [anchor]
     kept_frac = float(counts[args.warmup:, kept_layers].sum() / (args.steps * len(kept_layers) * nvs.sum()))
@@ -606,14 +621,10 @@ def e2e_leg(args, r, vp, ctx, dev, q_host, ks, vs_, kc, vc, span, budget, cap, w
     t0 = time.perf_counter()
     for s in range(args.warmup, S):
         one(s)
-    el = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([el], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        el = float(t.item())
+    el = max_over_ranks(time.perf_counter() - t0, world, dev)
     h2d = sum(t[0].numel() * t.element_size() for t in (qh, kvh, tlh))
     d2h = sum(t.numel() * t.element_size() for t in (out, kept, count, mass, stats))
-    return {"value": world * args.steps / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
+    return {"value": job_rate(world, args.steps, el), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": el * 1e3 / args.steps,
             "note": "host wall clock per step: pinned-host inputs copied in, the step's CUDA graph (K/V appends "
                     "+ 28 vp_decode_step calls captured through the C ABI) replayed, results copied back, "
