@@ -88,13 +88,15 @@ struct StepParams {
   int nk, nk_max;     // gather chunks used by this call / allocated
   int nm;             // gather CTAs that also merge a slice of the text partials (0: ns == 1)
   int nc;             // gather CTAs per (sequence, kv-head) = max(nk, nm)
-  int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= 256)
+  int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= kSliceMaxKept)
   int split_w;        // weight of one score split (bulk-tensor kernel)
 };
 
 // ---------------------------------------------------------------- host planning
 
 constexpr int kNkMax = 64;    // kept chunks per (sequence, kv-head)
+constexpr int kGmMaxChunk = 2048;   // kept rows of one chunk of the chunk gather
+constexpr int kSliceMaxKept = 256;  // kept rows per (sequence, kv-head) the slice gather holds
 constexpr int kTcRows = 128;  // rows of a tile of the tensor-core score kernel
 constexpr int kTcMaxBoxes = 384;  // page ids per cache a tensor-core score CTA stages
 constexpr int kNsMax = 256;   // score splits per (sequence, kv-head)
@@ -146,7 +148,7 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   // Kept chunks of about 2048 rows, smaller (down to 256) while the gather
   // grid would not fill the GPU once (measured against 1024-row chunks and a
   // twice-filled grid: the chunk gather 5% to 22% faster across the sweep).
-  long long nk = (kept_cap + 2047) / 2048;
+  long long nk = (kept_cap + kGmMaxChunk - 1) / kGmMaxChunk;
   const long long nk_want = (slots + units - 1) / units, nk_small = (kept_cap + 255) / 256;
   if (nk < nk_want) nk = nk_want < nk_small ? nk_want : nk_small;
   if (nk < 1) nk = 1;
@@ -161,7 +163,7 @@ inline Plan make_plan(int batch, int Hkv, int D, int num_sms, int max_visual, in
   }
   // Small kept sets of few sequences: one CTA per 16 output dimensions, so
   // that the whole gather is one short wave; otherwise one CTA per chunk.
-  const int gslice = kept_cap <= 256 && units * (D / 16) <= slots ? 1 : 0;
+  const int gslice = kept_cap <= kSliceMaxKept && units * (D / 16) <= slots ? 1 : 0;
   const int split_w = (int)((w_max + ns - 1) / ns);
   return Plan{(int)ns, cl, (int)nk, nm, (int)(nk > nm ? nk : nm), gslice, split_w};
 }

@@ -1175,7 +1175,6 @@ constexpr int kTcThreads = 192;
 
 template <int NS>
 struct TcCfgT {
-  static constexpr int SLOTS = NS;
   static constexpr int HALF = kTcRows * 128;           // 128 rows x 64 dimensions, swizzled
   static constexpr int SLOT = 2 * HALF;                // a 128 x 128 tile of K or of V
   static constexpr int QHALF = 16 * 128;               // 16 rows x 64 elements
@@ -2714,7 +2713,6 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // ---------------------------------------------------------------------------
 constexpr int kGmWarps = 4;
 constexpr int kGmSlots = 3;
-constexpr int kGmMaxChunk = 2048;  // kept rows per CTA (the plan's chunks are at most this)
 
 template <int D, int NT, int S>
 struct GmCfg {
@@ -2983,7 +2981,6 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
 // slice of V, fetched in the same round trip as the token's logits) and
 // combines both parts in log-sum-exp form.  No partial leaves the CTA.
 // ---------------------------------------------------------------------------
-constexpr int kSliceMaxKept = 256;
 constexpr int kSliceDims = 16;
 
 template <int GM>

@@ -1,0 +1,68 @@
+// Host-only check of the launch planner (make_plan, ws_layout): over a grid of
+// shapes, every plan covers the whole cache with its score splits, stays inside
+// the workspace the context allocated, keeps every gather chunk within the
+// chunk kernel's limit and picks the slice gather only for kept sets it holds.
+// Prints one line per violation and exits non-zero if there was any.
+#include <cstdio>
+
+#include "vp_internal.h"
+
+namespace {
+
+int fails = 0;
+
+void check(bool ok, const char* what, int B, int Hkv, int D, int sms, int mv, int ms, int cap, int tc, int gran) {
+  if (ok) return;
+  if (++fails <= 20)
+    std::printf("FAIL %s: B=%d Hkv=%d D=%d sms=%d max_visual=%d max_seq=%d kept_cap=%d tc=%d gran=%d\n", what, B, Hkv,
+                D, sms, mv, ms, cap, tc, gran);
+}
+
+bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+
+}  // namespace
+
+int main() {
+  using namespace vp;
+  const int Bs[] = {1, 2, 3, 7, 8, 32, 64, 100, 256};
+  const int Hkvs[] = {1, 2, 4, 8};
+  const int Ds[] = {64, 128};
+  const int SMs[] = {152, 148, 132, 1};
+  const int MVs[] = {0, 1, 576, 2304, 16384, 32767};
+  const int extra[] = {1, 513, 16384, 40000};
+  long long plans = 0;
+  for (int B : Bs)
+    for (int Hkv : Hkvs)
+      for (int D : Ds)
+        for (int sms : SMs)
+          for (int mv : MVs)
+            for (int ex : extra) {
+              const int ms = mv + ex, H = 7 * Hkv;
+              const WsLayout ws = ws_layout(B, H, Hkv, D, mv, ms, sms);
+              const int caps[] = {0, 1, 128, 129, 256, 257, 2048, 2049, mv, 100000};
+              for (int cap : caps)
+                for (int tc = 0; tc < 2; ++tc)
+                  for (int gran = 0; gran < 2; ++gran) {
+                    const Plan pl = make_plan(B, Hkv, D, sms, mv, ms, cap, gran, tc != 0);
+                    ++plans;
+                    const long long TR = tc ? kTcRows : 32;
+                    long long w_max = 2LL * ((ms + TR - 1) / TR) - mv / TR;
+                    if (w_max < 1) w_max = 1;
+#define CHECK(cond) check((cond), #cond, B, Hkv, D, sms, mv, ms, cap, tc, gran)
+                    CHECK(pl.ns >= 1 && pl.ns <= kNsMax);
+                    CHECK(pl.split_w >= 1 && (long long)pl.ns * pl.split_w >= w_max);
+                    CHECK(pl.ns <= ws.nsp_max);
+                    CHECK(pl.nk >= 1 && pl.nk <= kNkMax && pl.nk <= ws.nk_max);
+                    const int kmax = cap < mv ? cap : mv;
+                    CHECK((kmax + pl.nk - 1) / pl.nk <= kGmMaxChunk);
+                    CHECK((pl.ns == 1) == (pl.nm == 0));
+                    CHECK(pl.nm == 0 || (pow2(pl.nm) && pl.nm <= D / 16 && pl.nm <= kMaxMerge && pl.nm <= pl.nk));
+                    CHECK(pl.nc == (pl.nk > pl.nm ? pl.nk : pl.nm));
+                    CHECK(!pl.gslice || cap <= kSliceMaxKept);
+                    CHECK(pl.cl == 1 || pl.cl == 2 || pl.cl == 4 || pl.cl == 8);
+#undef CHECK
+                  }
+            }
+  std::printf("%lld plans, %d violations\n", plans, fails);
+  return fails ? 1 : 0;
+}
