@@ -164,13 +164,20 @@ class ClockSampler:
             return {"error": self.err or "NVML unavailable"}
         self._stop.set()
         self._t.join()
-        busy = [s for s in self.samples if not (s[1] & 0x1)] or self.samples
+        return self.summarize(self.samples, self.max_mhz)
+
+    @classmethod
+    def summarize(cls, samples, max_mhz):
+        """(SM MHz, reason bits) samples -> the JSON `clocks` object: the median
+        clock and the union of the active reasons over the samples taken while
+        the GPU was busy (all samples if it never was)."""
+        busy = [s for s in samples if not (s[1] & 0x1)] or samples
         seen = 0
         for _, r in busy:
             seen |= r
-        names = [n for bit, n in self.REASONS.items() if seen & bit and bit != 0x1]
+        names = [n for bit, n in cls.REASONS.items() if seen & bit and bit != 0x1]
         return {"sm_mhz": statistics.median(c for c, _ in busy) if busy else None,
-                "sm_max_mhz": self.max_mhz, "reasons": names, "samples": len(busy),
+                "sm_max_mhz": max_mhz, "reasons": names, "samples": len(busy),
                 "source": "NVML, 2 ms sampling during the timed region"}
 
 
