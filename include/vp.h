@@ -248,13 +248,22 @@ vp_status vp_compact_kv(vp_ctx* ctx, int32_t batch, const vp_kv* src, const vp_k
 typedef enum { VP_SCORE_AUTO = 0, VP_SCORE_MMA = 1, VP_SCORE_TC = 2 } vp_score_path;
 vp_status vp_set_score_path(vp_ctx* ctx, int32_t path);
 
+/* Launch record of the last successful vp_decode_step or vp_decode_gather
+ * call on this context, for profiling (an implementation detail with no
+ * counterpart in the paper): *score_path = VP_SCORE_TC when the tcgen05 score
+ * kernel ran, else VP_SCORE_MMA (the mma.sync, fallback or fp32 kernels);
+ * *kernels = the number of kernels the call enqueued.  Both are 0 before the
+ * first call.  Either pointer may be NULL.  Host only, no CUDA call. */
+vp_status vp_last_launch(const vp_ctx* ctx, int32_t* score_path, int32_t* kernels);
+
 /* Largest K_t the budget can produce for n_visual tokens (the kept_cap a
  * caller must provide); -1 for an invalid budget.  Host only, no CUDA. */
 int32_t vp_max_kept(const vp_budget* budget, int32_t n_visual);
 
 /* Text of the last error on this context ("" if none).  Valid until the next
- * call on the context.  Accepts NULL (returns the text of the last vp_init
- * failure in this thread). */
+ * call on the context.  Accepts NULL: then returns the text of the last
+ * failure in this thread of a call that takes no context (vp_init or
+ * vp_decode_step_noalloc), "" if that call succeeded. */
 const char* vp_last_error(const vp_ctx* ctx);
 
 /* Synchronises `cuda_stream`, then reads and clears the device error word.
@@ -298,7 +307,10 @@ vp_status vp_timing_read(vp_ctx* ctx, float* ms, int32_t max_slots, int32_t* n_s
  *     on different streams, or from several threads -- race and corrupt each
  *     other's results; serialise them;
  *   - device-side range checks still clamp bad spans and skip bad page ids,
- *     but their flags are not reported (there is no context to read them).
+ *     but their flags are not reported (there is no context to read them);
+ *   - on failure the reason (for VP_ERR_CAPACITY, the scratch bytes the call
+ *     would need) is readable through vp_last_error(NULL) in the calling
+ *     thread.
  * No cudaMalloc, cudaFree or other allocating call is made. */
 vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch, const void* q,
                                  const vp_kv* k_cache, const vp_kv* v_cache,

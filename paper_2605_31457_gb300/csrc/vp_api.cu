@@ -39,11 +39,12 @@ struct vp_ctx {
   std::vector<cudaEvent_t> tev;  // stage-timing events, 4 per slot
   int32_t tslots = 0;
   int64_t tcalls = 0;
+  int32_t last_score_path = 0;  // vp_last_launch: score kernel and kernel count of the last call
+  int32_t last_kernels = 0;
 };
 
 namespace {
 
-thread_local std::string g_init_error;
 
 constexpr int64_t kPpm = 1000000;
 constexpr int kMaxVisual = 32768;  // score keys of one sequence fit in shared memory
@@ -52,7 +53,7 @@ constexpr int kMaxGroup = 16;
 
 vp_status fail(vp_ctx* ctx, vp_status st, const std::string& msg) {
   if (ctx) ctx->last_error = msg;
-  else g_init_error = msg;
+  else vp::context_free_error() = msg;
   return st;
 }
 
@@ -125,6 +126,11 @@ bool kv_ok(const vp_ctx* ctx, const vp_kv* kv, const char* name, std::string* wh
 }
 
 }  // namespace
+
+std::string& vp::context_free_error() {
+  static thread_local std::string msg;
+  return msg;
+}
 
 extern "C" {
 
@@ -292,11 +298,13 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: gather kernel launch", e);
   if (tev) e = cudaEventRecordWithFlags(tev[3], st, rec_flags);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: timing event", e);
+  ctx->last_score_path = p.use_tc ? VP_SCORE_TC : VP_SCORE_MMA;
+  ctx->last_kernels = 3;
   return VP_OK;
 }
 
 const char* vp_last_error(const vp_ctx* ctx) {
-  return ctx ? ctx->last_error.c_str() : g_init_error.c_str();
+  return ctx ? ctx->last_error.c_str() : vp::context_free_error().c_str();
 }
 
 vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
@@ -373,6 +381,8 @@ vp_status vp_decode_gather(vp_ctx* ctx, int32_t batch, const void* q,
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: score kernel launch", e);
   e = vp::launch_gather(p, st);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_gather: merge kernel launch", e);
+  ctx->last_score_path = VP_SCORE_MMA;
+  ctx->last_kernels = 2;
   return VP_OK;
 }
 
@@ -437,6 +447,13 @@ vp_status vp_set_score_path(vp_ctx* ctx, int32_t path) {
   if (path != VP_SCORE_AUTO && path != VP_SCORE_MMA && path != VP_SCORE_TC)
     return fail(ctx, VP_ERR_INVALID_ARG, "vp_set_score_path: path must be VP_SCORE_AUTO, VP_SCORE_MMA or VP_SCORE_TC");
   ctx->score_path = path;
+  return VP_OK;
+}
+
+vp_status vp_last_launch(const vp_ctx* ctx, int32_t* score_path, int32_t* kernels) {
+  if (!ctx) return VP_ERR_NOT_INITIALIZED;
+  if (score_path) *score_path = ctx->last_score_path;
+  if (kernels) *kernels = ctx->last_kernels;
   return VP_OK;
 }
 

@@ -6,7 +6,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
+
 namespace vp {
+
+// Text of the last failure of a call that has no context (vp_init,
+// vp_decode_step_noalloc) in this thread; vp_last_error(NULL) returns it.
+std::string& context_free_error();
 
 // Device error word bits (vp_check_errors reports them).
 enum : unsigned {

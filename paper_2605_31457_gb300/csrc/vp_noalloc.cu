@@ -27,18 +27,32 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[VP_NOALLOC_SCRA
 
 constexpr int kMaxDevices = 64;
 
+// Shapes a scratch layout was planned for.
+struct LayoutKey {
+  int batch = -1, H = 0, Hkv = 0, D = 0, max_visual = 0, max_seq = 0;
+  bool operator==(const LayoutKey& o) const {
+    return batch == o.batch && H == o.H && Hkv == o.Hkv && D == o.D && max_visual == o.max_visual &&
+           max_seq == o.max_seq;
+  }
+};
+
 struct DeviceSlot {
   bool ready = false;
   void* scratch = nullptr;  // device address of g_noalloc_scratch on this device
   int num_sms = 0;
+  // The last call's scratch layout (planning it walks every batch size), and
+  // the largest visual span the select kernel's shared memory was raised for.
+  LayoutKey key;
+  vp::WsLayout lay;
+  int configured_visual = -1;
 };
 
 std::mutex g_mu;
 DeviceSlot g_slots[kMaxDevices];
-thread_local std::string g_noalloc_error;  // last failure text, kept for debuggers
 
+// Failure text goes where vp_last_error(NULL) reads it, in this thread.
 vp_status fail(vp_status st, const std::string& msg) {
-  g_noalloc_error = msg;
+  vp::context_free_error() = msg;
   return st;
 }
 
@@ -93,7 +107,7 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
                                             const vp_budget* budget, void* out, int32_t* kept_idx,
                                             int32_t kept_cap, int32_t* kept_count, float* mass,
                                             float* mass_stats, void* cuda_stream) {
-  g_noalloc_error.clear();
+  vp::context_free_error().clear();
   if (!cfg || !budget) return fail(VP_ERR_INVALID_ARG, "vp_decode_step_noalloc: cfg and budget are required");
   const vp_config& c = *cfg;
   if (c.max_batch < 1 || c.num_q_heads < 1 || c.num_kv_heads < 1 || c.num_q_heads % c.num_kv_heads ||
@@ -110,8 +124,9 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
       budget->r_hi_ppm < 0 || budget->r_hi_ppm > 1000000 || budget->ratio_ppm < 0 || budget->ratio_ppm > 1000000 ||
       budget->fixed_k < 0 || (budget->granularity != 0 && budget->granularity != 1))
     return fail(VP_ERR_INVALID_ARG, "vp_decode_step_noalloc: malformed budget");
-  if (kept_cap < max_kept(*budget, c.max_visual))
-    return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: kept_cap below the largest budget");
+  if (kept_cap < 0 || kept_cap < max_kept(*budget, c.max_visual))
+    return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: kept_cap " + std::to_string(kept_cap) +
+                " is negative or below the largest budget " + std::to_string(max_kept(*budget, c.max_visual)));
   if (batch == 0) return VP_OK;
   if (!q || !out || !text_len || !visual_span || !visual_span->vis_start || !visual_span->vis_len || !kept_count ||
       !mass || (kept_cap > 0 && !kept_idx) || !k_cache || !v_cache || !k_cache->data || !v_cache->data)
@@ -132,19 +147,32 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   vp_status st = setup_device(dev, &slot);
   if (st != VP_OK) return st;
 
-  // Scratch layout for this call (the partial formats of a context's workspace).
+  // Scratch layout for this call (the partial formats of a context's
+  // workspace), planned again only when the shapes change.
   const int H = c.num_q_heads, Hkv = c.num_kv_heads, G = H / Hkv, D = c.head_dim;
-  const vp::WsLayout L = vp::ws_layout(batch, H, Hkv, D, c.max_visual, c.max_seq, slot->num_sms);
+  const LayoutKey key{batch, H, Hkv, D, c.max_visual, c.max_seq};
+  vp::WsLayout L;
+  bool configure = false;
+  {
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!(slot->key == key)) {
+      slot->lay = vp::ws_layout(batch, H, Hkv, D, c.max_visual, c.max_seq, slot->num_sms);
+      slot->key = key;
+    }
+    L = slot->lay;
+    configure = c.max_visual > slot->configured_visual;
+  }
   if (L.total > (size_t)VP_NOALLOC_SCRATCH_BYTES)
     return fail(VP_ERR_CAPACITY, "vp_decode_step_noalloc: this batch and cfg need " + std::to_string(L.total) +
                 " scratch bytes; the fixed scratch holds " + std::to_string((size_t)VP_NOALLOC_SCRATCH_BYTES));
+  if (configure) {  // kernel attributes: the select kernel's shared memory grows with max_visual
+    e = vp::configure_kernels(c.max_visual, H, L.nsp_max);
+    if (e != cudaSuccess) return fail(VP_ERR_CUDA, std::string("vp_decode_step_noalloc: ") + cudaGetErrorString(e));
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (c.max_visual > slot->configured_visual) slot->configured_visual = c.max_visual;
+  }
 
-  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   char* base = static_cast<char*>(slot->scratch);
-  e = cudaMemsetAsync(base, 0, L.zero_bytes, stream);
-  if (e == cudaSuccess) e = vp::configure_kernels(c.max_visual, H, L.nsp_max);
-  if (e != cudaSuccess) return fail(VP_ERR_CUDA, std::string("vp_decode_step_noalloc: ") + cudaGetErrorString(e));
-
   vp::StepParams p;
   memset(&p, 0, sizeof p);
   p.dtype = c.dtype;
@@ -179,8 +207,13 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   p.hp = L.hp;
   p.nsp_max = L.nsp_max;
   p.nk_max = L.nk_max;
-  vp::plan_step(p, slot->num_sms, kept_cap, budget->granularity);
-  e = vp::launch_score(p, stream);
+  if (!vp::plan_step(p, slot->num_sms, kept_cap, budget->granularity))
+    return fail(VP_ERR_UNSUPPORTED, "vp_decode_step_noalloc: no launch plan serves this call");
+
+  // Only now that every check has passed: clear the counters, then launch.
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  e = cudaMemsetAsync(base, 0, L.zero_bytes, stream);
+  if (e == cudaSuccess) e = vp::launch_score(p, stream);
   if (e == cudaSuccess) e = vp::launch_select(p, stream);
   if (e == cudaSuccess) e = vp::launch_gather(p, stream);
   if (e != cudaSuccess) return fail(VP_ERR_CUDA, std::string("vp_decode_step_noalloc: launch: ") + cudaGetErrorString(e));

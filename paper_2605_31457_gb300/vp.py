@@ -41,7 +41,7 @@ VP_SCORE_TC = 2
 
 EXPORTED = ("vp_init", "vp_decode_step", "vp_max_kept", "vp_last_error", "vp_check_errors",
             "vp_timing_enable", "vp_timing_read", "vp_free", "vp_decode_step_noalloc", "vp_decode_gather",
-            "vp_set_diagnostics", "vp_set_score_path", "vp_compact_kv")
+            "vp_set_diagnostics", "vp_set_score_path", "vp_compact_kv", "vp_last_launch")
 VP_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -87,6 +87,8 @@ lib.vp_compact_kv.argtypes = [_P, ctypes.c_int32, ctypes.POINTER(vp_kv), ctypes.
 lib.vp_compact_kv.restype = ctypes.c_int
 lib.vp_set_score_path.argtypes = [_P, ctypes.c_int32]
 lib.vp_set_score_path.restype = ctypes.c_int
+lib.vp_last_launch.argtypes = [_P, ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32)]
+lib.vp_last_launch.restype = ctypes.c_int
 lib.vp_max_kept.argtypes = [ctypes.POINTER(vp_budget), ctypes.c_int32]
 lib.vp_max_kept.restype = ctypes.c_int32
 lib.vp_last_error.argtypes = [_P]
@@ -187,6 +189,14 @@ def vp_set_diagnostics(ctx, delta, n_act=None, active_bits=None):
     """Turns on (or off, with both arrays None) the N_act(delta) count and the
     OR-accumulated activity bits of later vp_decode_step calls."""
     return _check(lib.vp_set_diagnostics(ctx, float(delta), _ptr(n_act), _ptr(active_bits)), ctx)
+
+
+def vp_last_launch(ctx):
+    """(score kernel, kernels enqueued) of the last decode call on ctx:
+    VP_SCORE_TC or VP_SCORE_MMA, and the launch count."""
+    path, n = ctypes.c_int32(0), ctypes.c_int32(0)
+    _check(lib.vp_last_launch(ctx, ctypes.byref(path), ctypes.byref(n)), ctx)
+    return path.value, n.value
 
 
 def vp_max_kept(budget: vp_budget, n_visual: int) -> int:

@@ -83,3 +83,23 @@ def test_null_context_and_null_free(lib):
 ])
 def test_max_kept_is_the_budget_upper_bound(lib, budget, n, want):
     assert lib.vp_max_kept(lib.make_budget(**budget), n) == want
+
+
+def test_noalloc_rejects_before_any_cuda_call(lib):
+    """Malformed host arguments of the allocation-free entry point are refused
+    before it touches the GPU, with the reason readable via vp_last_error(NULL)."""
+    b = lib.make_budget()
+    cfg = lib.make_config(1, 8, 2, 64, 0, 16)
+    st = lib.lib.vp_decode_step_noalloc(None, 1, None, None, None, None, None, ctypes.byref(b), None,
+                                        None, 0, None, None, None, None)
+    assert st == lib.VP_ERR_INVALID_ARG and "cfg" in lib.vp_last_error(None)
+    st = lib.lib.vp_decode_step_noalloc(ctypes.byref(cfg), 1, None, None, None, None, None, ctypes.byref(b), None,
+                                        None, -1, None, None, None, None)
+    assert st == lib.VP_ERR_CAPACITY and "negative" in lib.vp_last_error(None)
+    st = lib.lib.vp_decode_step_noalloc(ctypes.byref(cfg), 0, None, None, None, None, None, ctypes.byref(b), None,
+                                        None, 0, None, None, None, None)
+    assert st == lib.VP_OK and lib.vp_last_error(None) == ""
+
+
+def test_last_launch_needs_a_context(lib):
+    assert lib.lib.vp_last_launch(None, None, None) == lib.VP_ERR_NOT_INITIALIZED

@@ -249,24 +249,26 @@ def test_capacity_and_argument_errors(vp):
 # -------------------------------------------------------------- full sizes
 
 def test_qwen7b_full_size_layer(vp):
-    """The benchmarked workload (B = 1, 28/4 heads, 1296 visual + 2561 text,
-    bf16) at two decode steps of one layer: every output against the oracle."""
+    """The B = 1 decode (28/4 heads, 1296 visual + 2561 text, bf16) at four
+    decode steps of one layer, two of them after the first shift of the visual
+    focus (every 64 steps): every output against the oracle."""
     r = W.QWEN7B
-    t_cap = r.capacity(64)
+    t_cap = r.capacity(66)
     li = W.make_layer(r, 3, t_cap=t_cap)
-    qs = W.make_queries(r, 3, li, steps=64)
+    qs = W.make_queries(r, 3, li, steps=66)
     rep = {}
-    for step in (0, 63):
+    for step in (0, 63, 64, 65):   # 64, 65: past the first shift of the visual focus
         inp = Hn.make_inputs(r, 3, step, t_cap=t_cap, q_override=qs[step])
         Hn.check_all(vp, inp, r.budget, report=rep)
         Hn.check_all(vp, inp, W.ADAPTIVE_10PCT, report=rep)
 
 
 def test_serving_paged_full_size_layer(vp):
-    """Batched serving: B = 32, paged (page 16), 2304 visual, text 512..4096."""
+    """Batched serving: B = 32, paged (page 16), 2304 visual, text 512..4096,
+    visual mass spread over [0.01, 0.4]: every sequence against the oracle."""
     r = W.SERVING
     inp = Hn.make_inputs(r, 0, 0)
-    gpu = Hn.check_all(vp, inp, r.budget, seqs=range(0, 32, 3))
+    gpu = Hn.check_all(vp, inp, r.budget)
     assert len(set(gpu["count"][:, 0].tolist())) > 1, "budgets should differ across the batch"
 
 
@@ -279,7 +281,7 @@ def test_sweep_points(vp, nv):
 
 # ------------------------------------------------- full sizes, device-generated
 
-def _device_generated(vp, r, seqs, budgets, rep):
+def _device_generated(vp, r, seqs, budgets, rep, expect_tc=None):
     """One layer of `r` at full size, drawn by the benchmark's on-device
     generator and run in the launch configuration the benchmark times; the
     sampled sequences are copied to the host and checked against the oracle."""
@@ -310,6 +312,8 @@ def _device_generated(vp, r, seqs, budgets, rep):
             vp.vp_decode_step(ctx, B, q, vp.kv_contiguous(k), vp.kv_contiguous(v), span, tl, bd, out, kept,
                               cap, count, mass, stats)
             vp.vp_check_errors(ctx)
+            if expect_tc is not None:
+                assert (vp.vp_last_launch(ctx)[0] == vp.VP_SCORE_TC) == expect_tc
             torch.cuda.synchronize()
             gpu = dict(out=out[sel].float().cpu().numpy(), kept=kept[sel].cpu().numpy(),
                        count=count[sel].cpu().numpy(), mass=mass[sel].cpu().numpy(), stats=stats[sel].cpu().numpy())
@@ -320,17 +324,20 @@ def _device_generated(vp, r, seqs, budgets, rep):
 
 
 def test_long_reasoning_full_size_layer(vp):
-    """Long reasoning: B = 8, 4096 visual + 16384 text, lognormal key norms."""
+    """Long reasoning: B = 8, 4096 visual + 16384 text, lognormal key norms,
+    in the benchmark's launch configuration (tcgen05 score kernel): every
+    sequence against the oracle."""
     rep = {}
-    _device_generated(vp, W.LONG, (0, 5, 7), [W.LONG.budget], rep)
+    _device_generated(vp, W.LONG, range(8), [W.LONG.budget], rep, expect_tc=True)
     assert rep.get("max_out_err", 0) < 2e-2
 
 
 @pytest.mark.parametrize("nv", [6400, 16384])
 def test_sweep_points_full_size(vp, nv):
-    """The long visual spans of the sweep at full size (B = 64, 32/8 heads):
-    the adaptive budget and 5% / 50% retention (slice and chunk gathers)."""
+    """The long visual spans of the sweep at full size (B = 64, 32/8 heads),
+    every benchmarked point -- the adaptive budget and 1% / 5% / 20% / 50%
+    retention (slice and chunk gathers) -- plus top-p."""
     r = W.sweep_recipe(nv, W.ADAPTIVE_5PCT)
     rep = {}
-    _device_generated(vp, r, (0, 33, 63), [W.ADAPTIVE_5PCT, W.SWEEP_BUDGETS[1], W.SWEEP_BUDGETS[3],
-                                           dict(mode=O.TOP_P, tau=0.1, ratio_ppm=100_000)], rep)
+    _device_generated(vp, r, (0, 33, 63), [W.ADAPTIVE_5PCT, *W.SWEEP_BUDGETS[:4],
+                                           dict(mode=O.TOP_P, tau=0.1, ratio_ppm=100_000)], rep, expect_tc=True)
