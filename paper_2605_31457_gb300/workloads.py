@@ -222,14 +222,15 @@ QWEN7B = Recipe(
 
 
 # Per-sequence planted-key scales of the batched-serving workload: c_b puts
-# the head-max visual mass of plain attention (tau = 1) of sequence b, at the
-# first decode step of layer 0, at the target drawn by serving_draws()
-# (log-uniform in [0.01, 0.4]).  Written by tests/calibrate_serving.py, which
-# finds each c_b by bisection with the CPU oracle on the host-generated layer.
-SERVING_PLANTED_SCALE = (0.90451, 1.20585, 1.20968, 0.82528, 0.71007, 1.19502, 0.88018, 0.92635,
-                         1.20303, 1.06794, 1.06656, 1.12195, 0.85663, 1.12711, 0.89072, 0.74196,
-                         0.97827, 1.43568, 0.83579, 1.03869, 0.99093, 1.07275, 1.07051, 0.92194,
-                         1.20852, 1.03203, 0.97725, 1.03680, 0.96554, 1.13716, 1.14613, 0.92405)
+# the visual mass that sets sequence b's budget (the head-max of the
+# temperature-scaled mass at the workload's tau = 0.1) at the first decode
+# step of layer 0 at the target drawn by serving_draws() (log-uniform in
+# [0.01, 0.4]).  Written by tests/calibrate_serving.py, which finds each c_b
+# by bisection with the CPU oracle on the host-generated layer.
+SERVING_PLANTED_SCALE = (1.42711, 1.57979, 1.50723, 1.26233, 1.20460, 1.39935, 1.34273, 1.35763,
+                         1.46155, 1.40012, 1.38687, 1.30919, 1.23687, 1.47727, 1.46549, 1.23615,
+                         1.28423, 1.63120, 1.25340, 1.42354, 1.43298, 1.37269, 1.33983, 1.42035,
+                         1.51391, 1.46188, 1.29900, 1.35225, 1.39636, 1.40571, 1.48737, 1.37757)
 
 
 def serving_draws(seed=3, batch=32):

@@ -269,7 +269,7 @@ def test_serving_paged_full_size_layer(vp):
     r = W.SERVING
     inp = Hn.make_inputs(r, 0, 0)
     gpu = Hn.check_all(vp, inp, r.budget)
-    assert len(set(gpu["count"][:, 0].tolist())) > 1, "budgets should differ across the batch"
+    assert len(set(gpu["count"][:, 0].tolist())) >= 4, "budgets should differ across the batch"
 
 
 @pytest.mark.parametrize("nv", [576, 2304])
