@@ -95,6 +95,7 @@ struct StepParams {
   int nm;             // gather CTAs that also merge a slice of the text partials (0: ns == 1)
   int nc;             // gather CTAs per (sequence, kv-head) = max(nk, nm)
   int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= kSliceMaxKept)
+  int fused;          // 1: one kernel selects and gathers (see fused_select_gather_ok)
   int split_w;        // weight of one score split (bulk-tensor kernel)
 };
 
@@ -244,6 +245,25 @@ void encode_kv_maps(StepParams& p);
 // at most 16 query heads per kv-head, pages of at least 8 rows).
 inline bool tc_eligible(int dtype, int D, int G, int paged, int page_size) {
   return dtype == 0 && D == 128 && G >= 1 && G <= 16 && (!paged || page_size >= 8);
+}
+
+// Whether one kernel (select + slice gather) serves the call: the slice
+// gather would (few sequences, kept sets of at most kSliceMaxKept rows), the
+// budget is known before the selection (not top-p), no diagnostics are
+// asked for, at most 8 query heads share a kv-head, and the select cluster's
+// CTAs split the output dimensions of every kv-head evenly into slices of 16
+// to 64 dimensions, and the score keys of a sequence fit in the cut's
+// registers (eight per thread of 512: N_v <= 4096).
+inline bool fused_select_gather_ok(const StepParams& p, int kept_cap) {
+  if (!p.gslice || p.anchor || p.mode == 4 || p.n_act || p.act_bits || p.G > 8 || kept_cap > kSliceMaxKept ||
+      p.max_visual > 4096)
+    return false;
+  const int hunits = p.granularity ? 1 : p.Hkv;
+  if (p.cl % hunits) return false;
+  const int rpg = p.cl / hunits;
+  if (p.D % rpg) return false;
+  const int W = p.D / rpg;
+  return W >= 16 && W <= 64;
 }
 
 // Launch plan and copy descriptors of a decode step (p's shapes, inputs and

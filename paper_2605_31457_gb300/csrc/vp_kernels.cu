@@ -678,11 +678,19 @@ __device__ __forceinline__ float fexp2(float x) {
 }
 // exp2(a - m) by the hardware approximation, an empty term (a = -inf) giving 0.
 __device__ __forceinline__ float fexp2_rel(float a, float m) { return a == -CUDART_INF_F ? 0.f : fexp2(a - m); }
+// A tile of the K or V cache: every byte of it is read once per call, so it
+// is marked evict-first in L2, which keeps the workspace (logits, split
+// partials) and the kernels' other data resident while a step streams
+// gigabytes of cache through the 129 MB L2.
 __device__ __forceinline__ void tma_load_4d(unsigned dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
                                             uint64_t* bar) {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
   asm volatile(
-      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];\n"
-      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;\n"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar)),
+        "l"(pol)
       : "memory");
 }
 
@@ -1949,6 +1957,15 @@ __device__ __forceinline__ int block_excl_scan(int x, int* wsum_s) {
   return res;
 }
 
+// The cut of the Top-K set (Eq. 3) found by a radix select over score keys
+// (float bits of non-negative scores, which order like the scores).
+struct RadixCut {
+  uint32_t theta;    // keys above theta are kept
+  unsigned krem;     // keys equal to theta to keep (the lowest-index ones)
+  unsigned n_theta;  // keys equal to theta (last pass only)
+  bool whole;        // the cut fell on a bucket boundary: keep every key >= theta + 1
+};
+
 template <int NTH>
 __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepParams p) {
   constexpr int NW = NTH / 32;
@@ -2227,7 +2244,9 @@ __global__ void __launch_bounds__(NTH) k_select(const __grid_constant__ StepPara
   // 4. Radix select of the K-th largest key, 8 bits per pass from the top;
   //    lanes holding the same digit add to the histogram once per warp.  One
   //    barrier per pass: every warp scans the finished histogram itself, and
-  //    pass p clears the buffer of pass p - 2 for pass p + 1.
+  //    pass p clears the buffer of pass p - 2 for pass p + 1.  (The same cut
+  //    as radix_cut, written out here: at 1024 threads this kernel runs at the
+  //    64-register limit, and with the shared routine it spilled more.)
   uint32_t theta = 0;
   unsigned krem = 0, n_theta = 0;  // keys equal to theta: to keep, in total
   if (topp) {
@@ -3163,6 +3182,540 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
   }
 }
 
+// ---------------------------------------------------------------------------
+// k_selgat: the select kernel and the slice gather in one launch, for the
+// calls the slice gather serves (few sequences, kept sets of at most
+// kSliceMaxKept rows, at most 8 query heads per kv-head, a budget known in
+// advance).  Grid (cl, nsel, B) in clusters of cl CTAs of 512 threads, one
+// cluster per selection unit (a sequence, or a (sequence, kv-head) when
+// granularity = 1); CTA r of the cluster owns the output dimensions
+// [d0, d0 + W) of one kv-head g.
+//   1. Every CTA merges the split statistics of every head into M_h, L1_h
+//      and the masses (Eq. 5, Eq. 6); rank 0 also takes the head mean, the
+//      head max (Sec. 4.3) and the budget K_t (Eq. 7 + clamp).
+//   2. Every CTA requests the text partials of the score splits for its
+//      dimensions, scores its slice of the visual tokens (S_i of Eq. 2) into
+//      rank 0's shared memory meanwhile, then sums the text part.
+//   3. Rank 0 cuts the Top-K_t set (Eq. 3) by a radix select over the keys
+//      held in registers and compacts it, ascending, into the output and its
+//      shared memory; the other CTAs copy it over distributed shared memory.
+//   4. Every CTA stages the V slices and logits of the kept tokens in shared
+//      memory in one round trip, attends over them for its dimensions (P.V on
+//      the tensor cores for bf16 caches) and combines the result with the
+//      text part in log-sum-exp form.  Nothing but the results leaves the
+//      cluster; one launch and one dependency replace two, and only the
+//      selection itself lies between the score kernel and the kept rows'
+//      loads.
+// ---------------------------------------------------------------------------
+constexpr int kSgThreads = 512;
+constexpr int kSgWarps = kSgThreads / 32;
+constexpr int kSgMaxW = 64;  // output dimensions of one CTA, at most
+
+// Register-resident Top-K cut of the fused kernel (Eq. 3) over n <= 8 * NTH
+// score keys: thread t holds keys [8t, 8t + 8), valid while below n.  Keys
+// are float bits of scores in [0, 1] (clamped below 2^30 by the producer), so
+// the digits skip the two top bits: passes on bits 29-22, 21-14, 13-6, 5-0.
+// Each quarter of the warps counts into its own histogram (no atomics shared
+// across quarters); lane L of every warp then owns digits 255-8L ... 248-8L
+// of the summed counts.  The three histogram sets rotate as in radix_cut
+// (zero on entry; pass p clears the set of pass p + 1).
+constexpr int kCutKeys = 8;
+template <int NTH>
+__device__ __forceinline__ RadixCut radix_cut_regs(const uint32_t (&k)[kCutKeys], int nvalid, int K,
+                                                   unsigned (*hist)[4][256]) {
+  const int tid = threadIdx.x, lane = tid & 31, grp = (tid >> 5) & 3;
+  unsigned krem = (unsigned)K, n_theta = 0;
+  bool whole = false;
+  uint32_t prefix = 0, mask = 0;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = pass < 3 ? 22 - 8 * pass : 0;
+    const uint32_t dmask = pass < 3 ? 255u : 63u;
+    if (pass >= 2)
+      for (int i = tid; i < 4 * 256; i += NTH) (&hist[(pass + 1) % 3][0][0])[i] = 0;
+    unsigned* h = hist[pass % 3][grp];
+#pragma unroll
+    for (int j = 0; j < kCutKeys; ++j)
+      if (j < nvalid && (k[j] & mask) == prefix) atomicAdd(&h[(k[j] >> shift) & dmask], 1u);
+    __syncthreads();
+    unsigned cnt8[8], tot = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cnt8[j] = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint4* hp = reinterpret_cast<const uint4*>(hist[pass % 3][q] + 248 - 8 * lane);
+      const uint4 lo = hp[0], hi = hp[1];  // digits 248-8L .. 251-8L, 252-8L .. 255-8L
+      cnt8[0] += hi.w; cnt8[1] += hi.z; cnt8[2] += hi.y; cnt8[3] += hi.x;
+      cnt8[4] += lo.w; cnt8[5] += lo.z; cnt8[6] += lo.y; cnt8[7] += lo.x;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) tot += cnt8[j];
+    unsigned incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned nn = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += nn;
+    }
+    const unsigned excl = incl - tot;
+    const bool mine = excl < krem && krem <= incl;
+    unsigned dsel = 0, before = 0, cnt = 0;
+    if (mine) {
+      unsigned run = excl;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (run + cnt8[j] >= krem) { dsel = 255 - 8 * lane - j; before = run; cnt = cnt8[j]; break; }
+        run += cnt8[j];
+      }
+    }
+    const int src = max(__ffs(__ballot_sync(0xffffffffu, mine)) - 1, 0);
+    dsel = __shfl_sync(0xffffffffu, dsel, src);
+    before = __shfl_sync(0xffffffffu, before, src);
+    cnt = __shfl_sync(0xffffffffu, cnt, src);
+    krem -= before;
+    prefix |= dsel << shift;
+    mask |= dmask << shift;
+    if (pass == 3) n_theta = cnt;
+    if (pass < 3 && krem == cnt) {  // the whole bucket is kept
+      whole = true;
+      break;
+    }
+  }
+  return RadixCut{whole ? prefix - 1u : prefix, krem, n_theta, whole};
+}
+
+// Ascending compaction of the register-resident keys (see radix_cut_regs):
+// keys above c.theta plus the first c.krem keys equal to it (every key when
+// take_all), written to kept (global) and kept_s (shared memory).
+template <int NTH>
+__device__ __forceinline__ void compact_kept_regs(const uint32_t (&k)[kCutKeys], int nvalid, int K, bool take_all,
+                                                  const RadixCut& c, int* wsum_s, int32_t* kept, int* kept_s) {
+  const int i0 = kCutKeys * (int)threadIdx.x;
+  const bool ties = !take_all && !c.whole && c.krem < c.n_theta;
+  int n_eq = 0;
+  if (ties)
+#pragma unroll
+    for (int j = 0; j < kCutKeys; ++j) n_eq += j < nvalid && k[j] == c.theta;
+  const int eq_before = ties ? block_excl_scan(n_eq, wsum_s) : 0;
+  const unsigned krem = ties ? c.krem : 0xffffffffu;
+  unsigned selm = 0;
+  {
+    int r = eq_before;
+#pragma unroll
+    for (int j = 0; j < kCutKeys; ++j) {
+      const bool v = j < nvalid;
+      const bool sel = v && (take_all || k[j] > c.theta || (!c.whole && k[j] == c.theta && (unsigned)r < krem));
+      r += v && k[j] == c.theta;
+      selm |= (unsigned)sel << j;
+    }
+  }
+  int o = block_excl_scan(__popc(selm), wsum_s);
+#pragma unroll
+  for (int j = 0; j < kCutKeys; ++j)
+    if (((selm >> j) & 1u) && o < K) {
+      kept[o] = i0 + j;
+      kept_s[o] = i0 + j;
+      ++o;
+    }
+}
+
+constexpr int kSgKP = kSliceMaxKept + 1;  // float row pitch of the kept logits (rows in distinct banks)
+constexpr int kSgPB = kSliceMaxKept + 8;  // bf16 row pitch of the kept probabilities (likewise)
+
+template <int GM>
+struct SgSmem {
+  float hM[kMaxHeads], hInv[kMaxHeads], hMass[kMaxHeads], hMass1[kMaxHeads];
+  float hMt[GM], hLt[GM];        // text-only max and sum of this CTA's heads
+  alignas(16) unsigned hist[3][4][256];  // radix histograms: three rotating sets of four
+  int wsum[32];
+  int K;                         // the budget K_t (rank 0; the others copy it)
+  int kept[kSliceMaxKept];       // the kept list (rank 0; the others copy it)
+  float pz[GM][kSgKP];           // kept logits, then (fp32 caches) probabilities
+  __nv_bfloat16 pb[8][kSgPB];    // bf16 caches: probabilities, B operand of the tensor-core P.V
+  float red[kSgWarps][128];      // P.V partials of every warp
+  float4 to[GM * kSgMaxW / 4];   // text part of the output
+  float fin[GM][2];              // kept max, kept sum
+};
+
+constexpr int kSgTextSplits = 10;  // text split partials a thread requests ahead
+
+// Byte offset of 16-byte piece c of row j in a stage of 128-byte rows, the
+// pieces XOR-swizzled by the row so that ldmatrix reads hit distinct banks.
+__device__ __forceinline__ unsigned sg_swz(int j, int c) { return (unsigned)(j * 128 + ((c ^ (j & 7)) << 4)); }
+
+template <typename T, int D, int GM>
+__global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ StepParams p) {
+  constexpr int NTH = kSgThreads, NW = kSgWarps;
+  constexpr bool BF = sizeof(T) == 2;
+  // Dynamic: the N_v score keys (rank 0's copy is used); after the cut, the
+  // kept rows' V slices.
+  extern __shared__ __align__(16) uint32_t key_s[];
+  __shared__ SgSmem<GM> sm;
+
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
+  const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < 3 * 4 * 256; i += NTH) (&sm.hist[0][0][0])[i] = 0;
+  const Seq sq = load_seq(p, b, false);  // an input: read before the wait
+  const int G = p.G, H = p.H, ns = p.ns, nv = sq.nv;
+  // This CTA's output: kv-head g, dimensions [d0, d0 + W) (the plan makes
+  // the cluster split every kv-head evenly, W a multiple of 16).
+  const int rpg = p.granularity ? ncl : ncl / p.Hkv;
+  const int W = D / rpg;
+  const int g = p.granularity ? gsel : rank / rpg;
+  const int d0 = (rank % rpg) * W;
+  const int64_t hrow0 = (int64_t)b * H + g * G;
+  const int nsel = p.granularity ? p.Hkv : 1;
+  pdl_wait();
+  pdl_trigger();
+  const float inv_tau = p.inv_tau;
+
+  // This CTA's slice of the visual tokens; each thread's first logit row is
+  // requested now so that it arrives while the statistics are merged.
+  const int per = (nv + ncl - 1) / ncl;
+  const int i0 = min(nv, rank * per), i1 = min(nv, i0 + per);
+  const int hbeg = p.granularity ? gsel * G : 0;
+  const int hcnt = p.granularity ? G : H;
+  const bool vec = (hbeg & 3) == 0 && (hcnt & 3) == 0;
+  const bool pre = vec && hcnt <= 32 && i0 + tid < i1;
+  float4 zpre[8];
+  if (pre) {
+    const float4* zr = reinterpret_cast<const float4*>(p.z_ws + ((int64_t)b * p.max_visual + i0 + tid) * p.hp + hbeg);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) zpre[q] = 4 * q < hcnt ? __ldcg(zr + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+
+  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5,
+  //    Eq. 6), and for this CTA's heads the text-only max and sum.  Sixteen
+  //    lanes per head (two heads per warp); lane l16 folds splits l16,
+  //    l16 + 16, ..., four records requested at a time (one round trip for
+  //    up to 64 splits).
+  {
+    const float* stb = p.split_st + (int64_t)b * H * p.nsp_max * ST_N;
+    const int sub = lane >> 4, l16 = lane & 15;
+    for (int h0 = 2 * warp; h0 < H; h0 += 2 * NW) {
+      const int h = h0 + sub;
+      float m = -CUDART_INF_F, a1v = 0.f, atv = 0.f, a1t = 0.f, att = 0.f;
+      float mt = -CUDART_INF_F, lt = 0.f;  // text only
+      for (int s0 = l16; s0 < ns; s0 += 64) {
+        float4 x[4], y[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int s = s0 + 16 * k;
+          if (h < H && s < ns) {
+            const float4* r = reinterpret_cast<const float4*>(stb + ((int64_t)h * p.nsp_max + s) * ST_N);
+            x[k] = __ldcg(r);
+            y[k] = __ldcg(r + 1);
+          } else {
+            x[k] = y[k] = make_float4(-CUDART_INF_F, 0.f, 0.f, 0.f);
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float mn = fmaxf(m, fmaxf(x[k].x, y[k].x));
+          if (mn > m) {
+            const float f1 = exp2_rel(m, mn), ft = exp2_tau(m, mn, inv_tau);
+            a1v *= f1; a1t *= f1; atv *= ft; att *= ft;
+            m = mn;
+          }
+          a1v = fmaf(exp2_rel(y[k].x, m), y[k].y, a1v);
+          atv = fmaf(exp2_tau(y[k].x, m, inv_tau), y[k].z, atv);
+          a1t = fmaf(exp2_rel(x[k].x, m), x[k].y, a1t);
+          att = fmaf(exp2_tau(x[k].x, m, inv_tau), x[k].z, att);
+          if (x[k].x > mt) { lt *= exp2_rel(mt, x[k].x); mt = x[k].x; }
+          lt = fmaf(exp2_rel(x[k].x, mt), x[k].y, lt);
+        }
+      }
+      float M = m, Mt = mt;
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, o));
+      }
+      const float f1 = exp2_rel(m, M), ft = exp2_tau(m, M, inv_tau), fl = exp2_rel(mt, Mt);
+      float L1v = a1v * f1, Ltv = atv * ft, L1t = a1t * f1, Ltt = att * ft, Lt = lt * fl;
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+        L1v += __shfl_xor_sync(0xffffffffu, L1v, o);
+        Ltv += __shfl_xor_sync(0xffffffffu, Ltv, o);
+        L1t += __shfl_xor_sync(0xffffffffu, L1t, o);
+        Ltt += __shfl_xor_sync(0xffffffffu, Ltt, o);
+        Lt += __shfl_xor_sync(0xffffffffu, Lt, o);
+      }
+      if (l16 == 0 && h < H) {
+        const float L1 = L1v + L1t, Lta = Ltv + Ltt;
+        sm.hM[h] = M;
+        sm.hInv[h] = L1 > 0.f ? 1.f / L1 : 0.f;
+        sm.hMass[h] = Lta > 0.f ? Ltv / Lta : 0.f;
+        sm.hMass1[h] = L1 > 0.f ? L1v / L1 : 0.f;
+        if (h >= g * G && h < g * G + G) { sm.hMt[h - g * G] = Mt; sm.hLt[h - g * G] = Lt; }
+      }
+    }
+  }
+  __syncthreads();
+
+  // 2a. Text partials of the score splits for this CTA's dimensions, requested
+  //     now and summed after the importance pass: thread (element
+  //     e = (head, 4 dimensions), split group sg of four) takes splits
+  //     sg, sg + 4, ...
+  const int W4 = W / 4, NE = G * W4;  // NE <= 128: four threads per element
+  const int te = tid >> 2, tsg = tid & 3;
+  const bool tlive = te < NE;
+  const int th = tlive ? te / W4 : 0, tdim = d0 + 4 * (tlive ? te % W4 : 0);
+  const float* tst = p.split_st + (hrow0 + th) * p.nsp_max * ST_N + ST_MT;
+  const float* tso = p.split_o + (hrow0 + th) * p.nsp_max * D + tdim;
+  float tmx[kSgTextSplits];
+  float4 tov[kSgTextSplits];
+#pragma unroll
+  for (int k = 0; k < kSgTextSplits; ++k) {
+    const int s = tsg + 4 * k;
+    const bool ok = tlive && s < ns;
+    tmx[k] = ok ? __ldcg(tst + (int64_t)s * ST_N) : -CUDART_INF_F;
+    tov[k] = ok ? __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D)) : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+
+  // Rank 0: head mean, head max (Sec. 4.3) and the budget (Eq. 7), on the
+  // last warp (whose importance rows come last).
+  if (rank == 0) {
+    if (warp == NW - 1) {
+      float smn = 0.f, mx = 0.f, s1 = 0.f;
+      for (int h = lane; h < H; h += 32) {
+        smn += sm.hMass[h];
+        mx = fmaxf(mx, sm.hMass[h]);
+        s1 += sm.hMass1[h];
+      }
+      smn = warp_sum(smn);
+      mx = warp_max(mx);
+      s1 = warp_sum(s1);
+      if (lane == 0) {
+        const int K = min(budget_k(p, mx, nv), min(p.kept_cap, kSliceMaxKept));
+        sm.K = K;
+        p.kept_count[(int64_t)b * nsel + gsel] = K;
+        if (gsel == 0 && p.mass_stats) {
+          float* ms = p.mass_stats + (int64_t)b * 4;
+          ms[0] = smn / H; ms[1] = mx; ms[2] = s1 / H; ms[3] = (float)K;
+        }
+      }
+    } else if (gsel == 0) {
+      for (int h = tid; h < H; h += NTH - 32) p.mass[(int64_t)b * H + h] = sm.hMass[h];
+    }
+  }
+
+  // 2b. Importance S_i (Eq. 2) of this CTA's slice, as float bits (S >= 0
+  //     orders like its bits), into rank 0's key array.
+  const float inv_cnt = 1.f / (float)hcnt;
+  uint32_t* key0 = ncl > 1 ? cluster.map_shared_rank(key_s, 0) : key_s;
+  unsigned bad = 0;
+  for (int i = i0 + tid; i < i1; i += NTH) {
+    const float* zr = p.z_ws + ((int64_t)b * p.max_visual + i) * p.hp + hbeg;
+    float a = 0.f;
+    if (pre && i == i0 + tid) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (4 * q < hcnt) {
+          const int h = hbeg + 4 * q;
+          a = fmaf(fexp2_rel(zpre[q].x, sm.hM[h]), sm.hInv[h], a);
+          a = fmaf(fexp2_rel(zpre[q].y, sm.hM[h + 1]), sm.hInv[h + 1], a);
+          a = fmaf(fexp2_rel(zpre[q].z, sm.hM[h + 2]), sm.hInv[h + 2], a);
+          a = fmaf(fexp2_rel(zpre[q].w, sm.hM[h + 3]), sm.hInv[h + 3], a);
+        }
+      }
+    } else if (vec) {
+      for (int hh = 0; hh < hcnt; hh += 4) {
+        const float4 z4 = __ldcg(reinterpret_cast<const float4*>(zr + hh));
+        const int h = hbeg + hh;
+        a = fmaf(fexp2_rel(z4.x, sm.hM[h]), sm.hInv[h], a);
+        a = fmaf(fexp2_rel(z4.y, sm.hM[h + 1]), sm.hInv[h + 1], a);
+        a = fmaf(fexp2_rel(z4.z, sm.hM[h + 2]), sm.hInv[h + 2], a);
+        a = fmaf(fexp2_rel(z4.w, sm.hM[h + 3]), sm.hInv[h + 3], a);
+      }
+    } else {
+      for (int hh = 0; hh < hcnt; ++hh)
+        a = fmaf(fexp2_rel(__ldcg(zr + hh), sm.hM[hbeg + hh]), sm.hInv[hbeg + hh], a);
+    }
+    const float sc = a * inv_cnt;
+    if (!isfinite(sc)) bad = 1;
+    key0[i] = min(__float_as_uint(sc), 0x3fffffffu);  // scores lie in [0, 1]: the top two bits are zero
+  }
+  if (bad) atomicOr(p.err, ERR_NONFINITE);
+
+  // 2c. The text part: sum exp2(m_s - m_text) * o_s over the splits, then over
+  //     the element's four split groups.
+  {
+    const float tmh = sm.hMt[th];
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < kSgTextSplits; ++k) {
+      const float w = exp2_rel(tmx[k], tmh);
+      a.x = fmaf(w, tov[k].x, a.x); a.y = fmaf(w, tov[k].y, a.y); a.z = fmaf(w, tov[k].z, a.z); a.w = fmaf(w, tov[k].w, a.w);
+    }
+    for (int s = tsg + 4 * kSgTextSplits; tlive && s < ns; s += 4) {
+      const float w = exp2_rel(__ldcg(tst + (int64_t)s * ST_N), tmh);
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D));
+      a.x = fmaf(w, v.x, a.x); a.y = fmaf(w, v.y, a.y); a.z = fmaf(w, v.z, a.z); a.w = fmaf(w, v.w, a.w);
+    }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+      a.x += __shfl_xor_sync(0xffffffffu, a.x, o);
+      a.y += __shfl_xor_sync(0xffffffffu, a.y, o);
+      a.z += __shfl_xor_sync(0xffffffffu, a.z, o);
+      a.w += __shfl_xor_sync(0xffffffffu, a.w, o);
+    }
+    if (tlive && tsg == 0) sm.to[te] = a;
+  }
+  if (ncl > 1) cluster.sync();  // rank 0 now sees every key
+  else __syncthreads();
+
+  // 3. Rank 0: the Top-K_t cut (Eq. 3) and the ascending compaction, with
+  //    every thread's eight keys in registers, into the output and into its
+  //    shared memory.
+  if (rank == 0) {
+    const int K = sm.K;
+    int32_t* kept = p.kept_idx + ((int64_t)b * nsel + gsel) * p.kept_cap;
+    const bool take_all = K >= nv;
+    const int nvalid = min(max(nv - kCutKeys * tid, 0), kCutKeys);
+    uint32_t kr[kCutKeys];
+    {
+      const uint4* kp = reinterpret_cast<const uint4*>(key_s + kCutKeys * tid);
+      const uint4 a = nvalid > 0 ? kp[0] : make_uint4(0u, 0u, 0u, 0u);
+      const uint4 c = nvalid > 4 ? kp[1] : make_uint4(0u, 0u, 0u, 0u);
+      kr[0] = a.x; kr[1] = a.y; kr[2] = a.z; kr[3] = a.w; kr[4] = c.x; kr[5] = c.y; kr[6] = c.z; kr[7] = c.w;
+    }
+    RadixCut cut{0u, (unsigned)K, 0u, false};
+    if (K > 0 && !take_all) cut = radix_cut_regs<NTH>(kr, nvalid, K, sm.hist);
+    if (K > 0) compact_kept_regs<NTH>(kr, nvalid, K, take_all, cut, sm.wsum, kept, sm.kept);
+    for (int i = max(K, 0) + tid; i < p.kept_cap; i += NTH) kept[i] = -1;
+  }
+  if (ncl > 1) cluster.sync();  // rank 0 holds the kept list
+  else __syncthreads();
+  // Every CTA copies the budget and the kept list from rank 0, then lets
+  // rank 0 go: its shared memory may be released once every CTA of the
+  // cluster has arrived (the matching wait is the kernel's last instruction).
+  int K;
+  if (ncl > 1) {
+    K = *cluster.map_shared_rank(&sm.K, 0);
+    if (rank != 0 && tid < K) sm.kept[tid] = cluster.map_shared_rank(&sm.kept[0], 0)[tid];
+    asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
+    __syncthreads();
+  } else {
+    K = sm.K;
+  }
+
+  // 4. Kept rows: this CTA's V slices to shared memory (asynchronous 16-byte
+  //    copies; bf16 rows of 128 bytes with swizzled pieces, fp32 rows packed)
+  //    and their logits, fetched together.  Rows past K, and rows whose
+  //    index or page is bad, are zero.
+  unsigned char* vst = reinterpret_cast<unsigned char*>(key_s);  // the keys are no longer read
+  const int CPR = W * (int)sizeof(T) / 16;                       // 16-byte pieces of a row slice
+  const int K16 = (K + 15) & ~15;
+  unsigned err = 0;
+  for (int i = tid; i < (BF ? K16 : K) * CPR; i += NTH) {
+    const int j = i / CPR, c = i % CPR;
+    const unsigned off = BF ? sg_swz(j, c) : (unsigned)((j * CPR + c) * 16);
+    const T* vr = nullptr;
+    if (j < K) {
+      const int id = sm.kept[j];
+      if (id >= 0 && id < nv) {
+        vr = kv_row<T>(p.v, p, b, g, sq.vs + id);
+        if (!vr) err |= ERR_PAGE;
+      } else {
+        err |= ERR_KEPT;
+      }
+    }
+    if (vr) cp_async16(smem_u32(vst + off), reinterpret_cast<const char*>(vr + d0) + 16 * c);
+    else *reinterpret_cast<uint4*>(vst + off) = make_uint4(0u, 0u, 0u, 0u);
+  }
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+  for (int i = tid; i < K * G; i += NTH) {
+    const int j = i / G, h = i % G;
+    const int id = sm.kept[j];
+    sm.pz[h][j] = (id >= 0 && id < nv) ? __ldcg(p.z_ws + ((int64_t)b * p.max_visual + id) * p.hp + g * G + h)
+                                       : -CUDART_INF_F;
+  }
+  __syncthreads();
+  // Per head: kept max, probabilities, sum.  bf16 caches: the probabilities
+  // as bf16 (the tensor-core operand), zero past K and for heads past G.
+  for (int h = warp; h < (BF ? 8 : G); h += NW) {
+    if (h >= G) {
+      for (int t = lane; t < K16; t += 32) sm.pb[h][t] = __float2bfloat16_rn(0.f);
+      continue;
+    }
+    float m = -CUDART_INF_F;
+    for (int t = lane; t < K; t += 32) m = fmaxf(m, sm.pz[h][t]);
+    m = warp_max(m);
+    float l = 0.f;
+    for (int t = lane; t < (BF ? K16 : K); t += 32) {
+      const float e = t < K ? exp2_rel(sm.pz[h][t], m) : 0.f;
+      if constexpr (BF) sm.pb[h][t] = __float2bfloat16_rn(e);
+      else sm.pz[h][t] = e;
+      l += e;
+    }
+    l = warp_sum(l);
+    if (lane == 0) { sm.fin[h][0] = m; sm.fin[h][1] = l; }
+  }
+  asm volatile("cp.async.wait_all;\n" ::: "memory");
+  __syncthreads();
+
+  // P.V.  bf16: on the tensor cores, mma m16n8k16 with A = V^T (16
+  // dimensions x 16 kept rows, ldmatrix.trans from the stage) and B = P^T
+  // (16 kept rows x 8 heads); warp w owns the 16-dimension tile w % (W / 16)
+  // over every (16 / (W / 16))-th step of 16 kept rows.  fp32: thread (part,
+  // head, dimension) sums every parts-th kept row on the CUDA cores.
+  const int nmt = W / 16;
+  if constexpr (BF) {
+    const int mt = warp % nmt, kg = warp / nmt, ngr = NW / nmt;
+    const int gr = lane >> 2, tg = lane & 3;
+    const int vrow = (lane & 7) + 8 * (lane >> 4), vcol = 8 * ((lane >> 3) & 1);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int ks = kg; ks < K16 / 16; ks += ngr) {
+      const __nv_bfloat16* pr = &sm.pb[gr][16 * ks + 2 * tg];
+      const uint32_t b0 = *reinterpret_cast<const uint32_t*>(pr);
+      const uint32_t b1 = *reinterpret_cast<const uint32_t*>(pr + 8);
+      const int col = 16 * mt + vcol;
+      uint32_t a0, a1, a2, a3;
+      ldsm_x4_t(smem_u32(vst) + sg_swz(16 * ks + vrow, col >> 3), a0, a1, a2, a3);
+      mma_bf16(acc, a0, a1, a2, a3, b0, b1);
+    }
+    float* rw = sm.red[warp];
+    rw[(2 * tg) * 16 + gr] = acc[0];
+    rw[(2 * tg + 1) * 16 + gr] = acc[1];
+    rw[(2 * tg) * 16 + gr + 8] = acc[2];
+    rw[(2 * tg + 1) * 16 + gr + 8] = acc[3];
+  } else {
+    const int items = GM * W, parts = NTH / items;
+    const int part = tid / items, it = tid % items, h = it / W, d = it % W;
+    float a = 0.f;
+    if (part < parts && h < G) {
+      const float* vf = reinterpret_cast<const float*>(vst);
+      for (int j = part; j < K; j += parts) a = fmaf(sm.pz[h][j], vf[j * W + d], a);
+    }
+    (&sm.red[0][0])[tid] = a;
+  }
+  if (err) atomicOr(p.err, err);
+  __syncthreads();
+
+  // Combine (thread per (head, dimension)): kept part and text part in
+  // log-sum-exp form, normalised over the kept and text tokens only.
+  for (int i = tid; i < G * W; i += NTH) {
+    const int h = i / W, d = i % W;
+    float kv = 0.f;
+    if constexpr (BF) {
+      const int mt = d / 16, dd = d % 16;
+      for (int kg = 0; kg < NW / nmt; ++kg) kv += sm.red[kg * nmt + mt][h * 16 + dd];
+    } else {
+      const int items = GM * W;
+      for (int part = 0; part < NTH / items; ++part) kv += (&sm.red[0][0])[part * items + h * W + d];
+    }
+    const float4 t4 = sm.to[h * W4 + d / 4];
+    const float tv = (d & 3) == 0 ? t4.x : (d & 3) == 1 ? t4.y : (d & 3) == 2 ? t4.z : t4.w;
+    const float mk = sm.fin[h][0], lk = sm.fin[h][1], mt = sm.hMt[h], lt = sm.hLt[h];
+    const float M = fmaxf(mk, mt);
+    const float ak = exp2_rel(mk, M), at = exp2_rel(mt, M);
+    const float den = ak * lk + at * lt;
+    const float o = den > 0.f ? (ak * kv + at * tv) / den : 0.f;
+    reinterpret_cast<T*>(p.out)[(hrow0 + h) * D + d0 + d] = from_f<T>(o);
+  }
+  if (ncl > 1) asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
+}
+
 // ------------------------------------------------------------------ launching
 
 cudaError_t launch_ex(void (*kernel)(StepParams), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
@@ -3330,6 +3883,7 @@ cudaError_t launch_score(const StepParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
+  if (p.fused) return cudaSuccess;  // the select kernel gathered
   if (p.dtype == 0)
     return p.D == 128 ? launch_gather_td<__nv_bfloat16, 128>(p, st) : launch_gather_td<__nv_bfloat16, 64>(p, st);
   return p.D == 128 ? launch_gather_td<float, 128>(p, st) : launch_gather_td<float, 64>(p, st);
@@ -3348,8 +3902,29 @@ cudaError_t launch_compact(const CompactParams& c, cudaStream_t st) {
   return cudaLaunchKernelEx(&cfg, k_compact, c);
 }
 
+// Dynamic shared memory of k_selgat: the score keys, later the kept rows'
+// V slices (bf16: rows of 128 bytes; fp32: rows of up to 256 bytes).
+size_t selgat_smem_bytes(int max_visual, int dtype) {
+  const size_t keys = select_smem_bytes(max_visual);
+  const size_t stage = (size_t)kSliceMaxKept * (dtype == 0 ? 128 : kSgMaxW * 4);
+  return keys > stage ? keys : stage;
+}
+
+template <typename T, int D>
+cudaError_t launch_selgat_td(const StepParams& p, dim3 grid, size_t smem, cudaStream_t st) {
+  if (p.G <= 4) return launch_ex(k_selgat<T, D, 4>, grid, dim3(kSgThreads), smem, st, p.cl, p);
+  return launch_ex(k_selgat<T, D, 8>, grid, dim3(kSgThreads), smem, st, p.cl, p);
+}
+
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.cl, p.granularity ? p.Hkv : 1, p.B);
+  if (p.fused) {
+    const size_t smem = selgat_smem_bytes(p.max_visual, p.dtype);
+    if (p.dtype == 0)
+      return p.D == 128 ? launch_selgat_td<__nv_bfloat16, 128>(p, grid, smem, st)
+                        : launch_selgat_td<__nv_bfloat16, 64>(p, grid, smem, st);
+    return p.D == 128 ? launch_selgat_td<float, 128>(p, grid, smem, st) : launch_selgat_td<float, 64>(p, grid, smem, st);
+  }
   const size_t smem = select_smem_bytes(p.max_visual);
   if ((p.max_visual + p.cl - 1) / p.cl <= kSelSliceSmall) return launch_ex(k_select<512>, grid, dim3(512), smem, st, p.cl, p);
   return launch_ex(k_select<1024>, grid, dim3(1024), smem, st, p.cl, p);
@@ -3458,6 +4033,18 @@ cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {
     cudaFuncAttributes attr;
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k);
     if (e == cudaSuccess && attr.maxDynamicSharedSizeBytes < need) e = set_smem(k, need);
+  }
+  void (*const selgat[2][4])(StepParams) = {
+      {k_selgat<__nv_bfloat16, 128, 4>, k_selgat<__nv_bfloat16, 128, 8>, k_selgat<__nv_bfloat16, 64, 4>,
+       k_selgat<__nv_bfloat16, 64, 8>},
+      {k_selgat<float, 128, 4>, k_selgat<float, 128, 8>, k_selgat<float, 64, 4>, k_selgat<float, 64, 8>}};
+  for (int dt = 0; dt < 2; ++dt) {
+    const int need_sg = (int)selgat_smem_bytes(max_visual, dt);
+    for (void (*k)(StepParams) : selgat[dt]) {
+      cudaFuncAttributes attr;
+      if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k);
+      if (e == cudaSuccess && attr.maxDynamicSharedSizeBytes < need_sg) e = set_smem(k, need_sg);
+    }
   }
   return e == cudaSuccess ? configure_fixed_kernels() : e;
 }
