@@ -3368,8 +3368,32 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   pdl_trigger();
   const float inv_tau = p.inv_tau;
 
+  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5,
+  //    Eq. 6), and for this CTA's heads the text-only max and sum.  Sixteen
+  //    lanes per head (two heads per warp); lane l16 folds splits l16,
+  //    l16 + 16, ..., four records requested at a time (one round trip for
+  //    up to 64 splits).  The first round's records are requested before
+  //    anything else: they are on the critical path.
+  const float* stb = p.split_st + (int64_t)b * H * p.nsp_max * ST_N;
+  const int sub = lane >> 4, l16 = lane & 15;
+  auto fetch4 = [&](int h, int s0, float4 (&x)[4], float4 (&y)[4]) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int s = s0 + 16 * k;
+      if (h < H && s < ns) {
+        const float4* r = reinterpret_cast<const float4*>(stb + ((int64_t)h * p.nsp_max + s) * ST_N);
+        x[k] = __ldcg(r);
+        y[k] = __ldcg(r + 1);
+      } else {
+        x[k] = y[k] = make_float4(-CUDART_INF_F, 0.f, 0.f, 0.f);
+      }
+    }
+  };
+  float4 rx[4], ry[4];
+  fetch4(2 * warp + sub, l16, rx, ry);
+
   // This CTA's slice of the visual tokens; each thread's first logit row is
-  // requested now so that it arrives while the statistics are merged.
+  // requested next so that it arrives while the statistics are merged.
   const int per = (nv + ncl - 1) / ncl;
   const int i0 = min(nv, rank * per), i1 = min(nv, i0 + per);
   const int hbeg = p.granularity ? gsel * G : 0;
@@ -3383,71 +3407,53 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
     for (int q = 0; q < 8; ++q) zpre[q] = 4 * q < hcnt ? __ldcg(zr + q) : make_float4(0.f, 0.f, 0.f, 0.f);
   }
 
-  // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5,
-  //    Eq. 6), and for this CTA's heads the text-only max and sum.  Sixteen
-  //    lanes per head (two heads per warp); lane l16 folds splits l16,
-  //    l16 + 16, ..., four records requested at a time (one round trip for
-  //    up to 64 splits).
-  {
-    const float* stb = p.split_st + (int64_t)b * H * p.nsp_max * ST_N;
-    const int sub = lane >> 4, l16 = lane & 15;
-    for (int h0 = 2 * warp; h0 < H; h0 += 2 * NW) {
-      const int h = h0 + sub;
-      float m = -CUDART_INF_F, a1v = 0.f, atv = 0.f, a1t = 0.f, att = 0.f;
-      float mt = -CUDART_INF_F, lt = 0.f;  // text only
-      for (int s0 = l16; s0 < ns; s0 += 64) {
-        float4 x[4], y[4];
+  for (int h0 = 2 * warp; h0 < H; h0 += 2 * NW) {
+    const int h = h0 + sub;
+    if (h0 != 2 * warp) fetch4(h, l16, rx, ry);  // the first round's records are in flight already
+    float m = -CUDART_INF_F, a1v = 0.f, atv = 0.f, a1t = 0.f, att = 0.f;
+    float mt = -CUDART_INF_F, lt = 0.f;  // text only
+    for (int s0 = l16;; s0 += 64) {
+      if (s0 != l16) fetch4(h, s0, rx, ry);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int s = s0 + 16 * k;
-          if (h < H && s < ns) {
-            const float4* r = reinterpret_cast<const float4*>(stb + ((int64_t)h * p.nsp_max + s) * ST_N);
-            x[k] = __ldcg(r);
-            y[k] = __ldcg(r + 1);
-          } else {
-            x[k] = y[k] = make_float4(-CUDART_INF_F, 0.f, 0.f, 0.f);
-          }
+      for (int k = 0; k < 4; ++k) {
+        const float mn = fmaxf(m, fmaxf(rx[k].x, ry[k].x));
+        if (mn > m) {
+          const float f1 = exp2_rel(m, mn), ft = exp2_tau(m, mn, inv_tau);
+          a1v *= f1; a1t *= f1; atv *= ft; att *= ft;
+          m = mn;
         }
+        a1v = fmaf(exp2_rel(ry[k].x, m), ry[k].y, a1v);
+        atv = fmaf(exp2_tau(ry[k].x, m, inv_tau), ry[k].z, atv);
+        a1t = fmaf(exp2_rel(rx[k].x, m), rx[k].y, a1t);
+        att = fmaf(exp2_tau(rx[k].x, m, inv_tau), rx[k].z, att);
+        if (rx[k].x > mt) { lt *= exp2_rel(mt, rx[k].x); mt = rx[k].x; }
+        lt = fmaf(exp2_rel(rx[k].x, mt), rx[k].y, lt);
+      }
+      if (s0 + 64 >= ns) break;
+    }
+    float M = m, Mt = mt;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float mn = fmaxf(m, fmaxf(x[k].x, y[k].x));
-          if (mn > m) {
-            const float f1 = exp2_rel(m, mn), ft = exp2_tau(m, mn, inv_tau);
-            a1v *= f1; a1t *= f1; atv *= ft; att *= ft;
-            m = mn;
-          }
-          a1v = fmaf(exp2_rel(y[k].x, m), y[k].y, a1v);
-          atv = fmaf(exp2_tau(y[k].x, m, inv_tau), y[k].z, atv);
-          a1t = fmaf(exp2_rel(x[k].x, m), x[k].y, a1t);
-          att = fmaf(exp2_tau(x[k].x, m, inv_tau), x[k].z, att);
-          if (x[k].x > mt) { lt *= exp2_rel(mt, x[k].x); mt = x[k].x; }
-          lt = fmaf(exp2_rel(x[k].x, mt), x[k].y, lt);
-        }
-      }
-      float M = m, Mt = mt;
+    for (int o = 1; o < 16; o <<= 1) {
+      M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, o));
+    }
+    const float f1 = exp2_rel(m, M), ft = exp2_tau(m, M, inv_tau), fl = exp2_rel(mt, Mt);
+    float L1v = a1v * f1, Ltv = atv * ft, L1t = a1t * f1, Ltt = att * ft, Lt = lt * fl;
 #pragma unroll
-      for (int o = 1; o < 16; o <<= 1) {
-        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-        Mt = fmaxf(Mt, __shfl_xor_sync(0xffffffffu, Mt, o));
-      }
-      const float f1 = exp2_rel(m, M), ft = exp2_tau(m, M, inv_tau), fl = exp2_rel(mt, Mt);
-      float L1v = a1v * f1, Ltv = atv * ft, L1t = a1t * f1, Ltt = att * ft, Lt = lt * fl;
-#pragma unroll
-      for (int o = 1; o < 16; o <<= 1) {
-        L1v += __shfl_xor_sync(0xffffffffu, L1v, o);
-        Ltv += __shfl_xor_sync(0xffffffffu, Ltv, o);
-        L1t += __shfl_xor_sync(0xffffffffu, L1t, o);
-        Ltt += __shfl_xor_sync(0xffffffffu, Ltt, o);
-        Lt += __shfl_xor_sync(0xffffffffu, Lt, o);
-      }
-      if (l16 == 0 && h < H) {
-        const float L1 = L1v + L1t, Lta = Ltv + Ltt;
-        sm.hM[h] = M;
-        sm.hInv[h] = L1 > 0.f ? 1.f / L1 : 0.f;
-        sm.hMass[h] = Lta > 0.f ? Ltv / Lta : 0.f;
-        sm.hMass1[h] = L1 > 0.f ? L1v / L1 : 0.f;
-        if (h >= g * G && h < g * G + G) { sm.hMt[h - g * G] = Mt; sm.hLt[h - g * G] = Lt; }
-      }
+    for (int o = 1; o < 16; o <<= 1) {
+      L1v += __shfl_xor_sync(0xffffffffu, L1v, o);
+      Ltv += __shfl_xor_sync(0xffffffffu, Ltv, o);
+      L1t += __shfl_xor_sync(0xffffffffu, L1t, o);
+      Ltt += __shfl_xor_sync(0xffffffffu, Ltt, o);
+      Lt += __shfl_xor_sync(0xffffffffu, Lt, o);
+    }
+    if (l16 == 0 && h < H) {
+      const float L1 = L1v + L1t, Lta = Ltv + Ltt;
+      sm.hM[h] = M;
+      sm.hInv[h] = L1 > 0.f ? 1.f / L1 : 0.f;
+      sm.hMass[h] = Lta > 0.f ? Ltv / Lta : 0.f;
+      sm.hMass1[h] = L1 > 0.f ? L1v / L1 : 0.f;
+      if (h >= g * G && h < g * G + G) { sm.hMt[h - g * G] = Mt; sm.hLt[h - g * G] = Lt; }
     }
   }
   __syncthreads();
@@ -3599,14 +3605,22 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
     K = sm.K;
   }
 
-  // 4. Kept rows: this CTA's V slices to shared memory (asynchronous 16-byte
-  //    copies; bf16 rows of 128 bytes with swizzled pieces, fp32 rows packed)
-  //    and their logits, fetched together.  Rows past K, and rows whose
-  //    index or page is bad, are zero.
+  // 4. Kept rows: their logits and this CTA's V slices to shared memory
+  //    (asynchronous copies; V in 16-byte pieces, bf16 rows of 128 bytes with
+  //    swizzled pieces, fp32 rows packed), all requested together.  Rows past
+  //    K, and rows whose index or page is bad, are zero.
   unsigned char* vst = reinterpret_cast<unsigned char*>(key_s);  // the keys are no longer read
   const int CPR = W * (int)sizeof(T) / 16;                       // 16-byte pieces of a row slice
   const int K16 = (K + 15) & ~15;
   unsigned err = 0;
+  // Logits first (the older copy group: the softmax waits for it alone).
+  for (int i = tid; i < K * G; i += NTH) {
+    const int j = i / G, h = i % G;
+    const int id = sm.kept[j];
+    if (id >= 0 && id < nv) cp_async4(smem_u32(&sm.pz[h][j]), p.z_ws + ((int64_t)b * p.max_visual + id) * p.hp + g * G + h);
+    else sm.pz[h][j] = -CUDART_INF_F;
+  }
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
   for (int i = tid; i < (BF ? K16 : K) * CPR; i += NTH) {
     const int j = i / CPR, c = i % CPR;
     const unsigned off = BF ? sg_swz(j, c) : (unsigned)((j * CPR + c) * 16);
@@ -3624,12 +3638,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
     else *reinterpret_cast<uint4*>(vst + off) = make_uint4(0u, 0u, 0u, 0u);
   }
   asm volatile("cp.async.commit_group;\n" ::: "memory");
-  for (int i = tid; i < K * G; i += NTH) {
-    const int j = i / G, h = i % G;
-    const int id = sm.kept[j];
-    sm.pz[h][j] = (id >= 0 && id < nv) ? __ldcg(p.z_ws + ((int64_t)b * p.max_visual + id) * p.hp + g * G + h)
-                                       : -CUDART_INF_F;
-  }
+  asm volatile("cp.async.wait_group 1;\n" ::: "memory");
   __syncthreads();
   // Per head: kept max, probabilities, sum.  bf16 caches: the probabilities
   // as bf16 (the tensor-core operand), zero past K and for heads past G.
@@ -3651,7 +3660,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
     l = warp_sum(l);
     if (lane == 0) { sm.fin[h][0] = m; sm.fin[h][1] = l; }
   }
-  asm volatile("cp.async.wait_all;\n" ::: "memory");
+  asm volatile("cp.async.wait_group 0;\n" ::: "memory");  // the V rows
   __syncthreads();
 
   // P.V.  bf16: on the tensor cores, mma m16n8k16 with A = V^T (16
