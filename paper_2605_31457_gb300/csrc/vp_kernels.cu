@@ -3215,47 +3215,57 @@ constexpr int kSgMaxW = 64;  // output dimensions of one CTA, at most
 // score keys: thread t holds keys [8t, 8t + 8), valid while below n.  Keys
 // are float bits of scores in [0, 1] (clamped below 2^30 by the producer), so
 // the digits skip the two top bits: passes on bits 29-22, 21-14, 13-6, 5-0.
-// Each quarter of the warps counts into its own histogram (no atomics shared
-// across quarters); lane L of every warp then owns digits 255-8L ... 248-8L
-// of the summed counts.  The three histogram sets rotate as in radix_cut
-// (zero on entry; pass p clears the set of pass p + 1).
+// The first digits of the scores concentrate in few buckets, so every warp
+// counts into its own histogram (hist: two sets of NTH / 32 histograms of 256
+// bins in shared memory, alternating between passes; each warp clears its
+// own histogram of a set before counting into it); thread d < 256 then adds
+// up digit d over the warps into tot, and lane L of every warp owns digits
+// 255-8L ... 248-8L of the sums.
 constexpr int kCutKeys = 8;
 template <int NTH>
-__device__ __forceinline__ RadixCut radix_cut_regs(const uint32_t (&k)[kCutKeys], int nvalid, int K,
-                                                   unsigned (*hist)[4][256]) {
-  const int tid = threadIdx.x, lane = tid & 31, grp = (tid >> 5) & 3;
+__device__ __forceinline__ RadixCut radix_cut_regs(const uint32_t (&k)[kCutKeys], int nvalid, int K, unsigned* hist,
+                                                   unsigned* tot) {
+  constexpr int NW = NTH / 32;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   unsigned krem = (unsigned)K, n_theta = 0;
   bool whole = false;
   uint32_t prefix = 0, mask = 0;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = pass < 3 ? 22 - 8 * pass : 0;
     const uint32_t dmask = pass < 3 ? 255u : 63u;
-    if (pass >= 2)
-      for (int i = tid; i < 4 * 256; i += NTH) (&hist[(pass + 1) % 3][0][0])[i] = 0;
-    unsigned* h = hist[pass % 3][grp];
+    unsigned* h = hist + ((pass & 1) * NW + warp) * 256;
+    // This warp's histogram of the set: last read before the previous pass's
+    // second barrier, so it may be cleared now.
+    reinterpret_cast<uint4*>(h)[2 * lane] = make_uint4(0u, 0u, 0u, 0u);
+    reinterpret_cast<uint4*>(h)[2 * lane + 1] = make_uint4(0u, 0u, 0u, 0u);
+    __syncwarp();
 #pragma unroll
     for (int j = 0; j < kCutKeys; ++j)
       if (j < nvalid && (k[j] & mask) == prefix) atomicAdd(&h[(k[j] >> shift) & dmask], 1u);
     __syncthreads();
-    unsigned cnt8[8], tot = 0;
+    if (tid < 256) {
+      unsigned c = 0;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) cnt8[j] = 0;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint4* hp = reinterpret_cast<const uint4*>(hist[pass % 3][q] + 248 - 8 * lane);
-      const uint4 lo = hp[0], hi = hp[1];  // digits 248-8L .. 251-8L, 252-8L .. 255-8L
-      cnt8[0] += hi.w; cnt8[1] += hi.z; cnt8[2] += hi.y; cnt8[3] += hi.x;
-      cnt8[4] += lo.w; cnt8[5] += lo.z; cnt8[6] += lo.y; cnt8[7] += lo.x;
+      for (int w = 0; w < NW; ++w) c += hist[((pass & 1) * NW + w) * 256 + tid];
+      tot[tid] = c;
+    }
+    __syncthreads();
+    unsigned cnt8[8], sum8 = 0;
+    {
+      const uint4* tp = reinterpret_cast<const uint4*>(tot + 248 - 8 * lane);
+      const uint4 lo = tp[0], hi = tp[1];  // digits 248-8L .. 251-8L, 252-8L .. 255-8L
+      cnt8[0] = hi.w; cnt8[1] = hi.z; cnt8[2] = hi.y; cnt8[3] = hi.x;
+      cnt8[4] = lo.w; cnt8[5] = lo.z; cnt8[6] = lo.y; cnt8[7] = lo.x;
     }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) tot += cnt8[j];
-    unsigned incl = tot;
+    for (int j = 0; j < 8; ++j) sum8 += cnt8[j];
+    unsigned incl = sum8;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const unsigned nn = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += nn;
     }
-    const unsigned excl = incl - tot;
+    const unsigned excl = incl - sum8;
     const bool mine = excl < krem && krem <= incl;
     unsigned dsel = 0, before = 0, cnt = 0;
     if (mine) {
@@ -3324,7 +3334,7 @@ template <int GM>
 struct SgSmem {
   float hM[kMaxHeads], hInv[kMaxHeads], hMass[kMaxHeads], hMass1[kMaxHeads];
   float hMt[GM], hLt[GM];        // text-only max and sum of this CTA's heads
-  alignas(16) unsigned hist[3][4][256];  // radix histograms: three rotating sets of four
+  alignas(16) unsigned tot[256];  // radix: digit counts summed over the warps
   int wsum[32];
   int K;                         // the budget K_t (rank 0; the others copy it)
   int kept[kSliceMaxKept];       // the kept list (rank 0; the others copy it)
@@ -3353,7 +3363,6 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank(), ncl = (int)cluster.num_blocks();
   const int gsel = blockIdx.y, b = blockIdx.z, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int i = tid; i < 3 * 4 * 256; i += NTH) (&sm.hist[0][0][0])[i] = 0;
   const Seq sq = load_seq(p, b, false);  // an input: read before the wait
   const int G = p.G, H = p.H, ns = p.ns, nv = sq.nv;
   // This CTA's output: kv-head g, dimensions [d0, d0 + W) (the plan makes
@@ -3586,7 +3595,8 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
       kr[0] = a.x; kr[1] = a.y; kr[2] = a.z; kr[3] = a.w; kr[4] = c.x; kr[5] = c.y; kr[6] = c.z; kr[7] = c.w;
     }
     RadixCut cut{0u, (unsigned)K, 0u, false};
-    if (K > 0 && !take_all) cut = radix_cut_regs<NTH>(kr, nvalid, K, sm.hist);
+    __syncthreads();  // every key is in registers: the key array holds the warps' histograms from here on
+    if (K > 0 && !take_all) cut = radix_cut_regs<NTH>(kr, nvalid, K, key_s, sm.tot);
     if (K > 0) compact_kept_regs<NTH>(kr, nvalid, K, take_all, cut, sm.wsum, kept, sm.kept);
     for (int i = max(K, 0) + tid; i < p.kept_cap; i += NTH) kept[i] = -1;
   }
@@ -3911,12 +3921,15 @@ cudaError_t launch_compact(const CompactParams& c, cudaStream_t st) {
   return cudaLaunchKernelEx(&cfg, k_compact, c);
 }
 
-// Dynamic shared memory of k_selgat: the score keys, later the kept rows'
-// V slices (bf16: rows of 128 bytes; fp32: rows of up to 256 bytes).
+// Dynamic shared memory of k_selgat: the score keys, then the cut's per-warp
+// histograms, then the kept rows' V slices (bf16: rows of 128 bytes; fp32:
+// rows of up to 256 bytes).
 size_t selgat_smem_bytes(int max_visual, int dtype) {
   const size_t keys = select_smem_bytes(max_visual);
   const size_t stage = (size_t)kSliceMaxKept * (dtype == 0 ? 128 : kSgMaxW * 4);
-  return keys > stage ? keys : stage;
+  const size_t hist = (size_t)2 * kSgWarps * 256 * 4;  // the cut's per-warp histograms
+  size_t n = keys > stage ? keys : stage;
+  return n > hist ? n : hist;
 }
 
 template <typename T, int D>
