@@ -276,7 +276,7 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
     p.act_bits = ctx->diag_bits;
     p.act_words = (c.max_visual + 31) / 32;
   }
-  p.fused = vp::fused_select_gather_ok(p, kept_cap) ? 1 : 0;
+  p.fused = vp::select_kind(p, kept_cap);
 
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   cudaEvent_t* tev = nullptr;
@@ -300,7 +300,7 @@ vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
   if (tev) e = cudaEventRecordWithFlags(tev[3], st, rec_flags);
   if (e != cudaSuccess) return cuda_fail(ctx, "vp_decode_step: timing event", e);
   ctx->last_score_path = p.use_tc ? VP_SCORE_TC : VP_SCORE_MMA;
-  ctx->last_kernels = p.fused ? 2 : 3;
+  ctx->last_kernels = p.fused == 1 ? 2 : 3;
   return VP_OK;
 }
 

@@ -95,7 +95,8 @@ struct StepParams {
   int nm;             // gather CTAs that also merge a slice of the text partials (0: ns == 1)
   int nc;             // gather CTAs per (sequence, kv-head) = max(nk, nm)
   int gslice;         // 1: kept sets fit the single-pass slice gather (kept_cap <= kSliceMaxKept)
-  int fused;          // 1: one kernel selects and gathers (see fused_select_gather_ok)
+  int fused;          // select kernel: 0 k_select; 1 k_selgat, which also gathers (fused_select_gather_ok);
+                      // 2 k_selgat selecting only (fast_select_ok)
   int split_w;        // weight of one score split (bulk-tensor kernel)
 };
 
@@ -264,6 +265,17 @@ inline bool fused_select_gather_ok(const StepParams& p, int kept_cap) {
   if (p.D % rpg) return false;
   const int W = p.D / rpg;
   return W >= 16 && W <= 64;
+}
+
+// Whether the selection of a call the fused kernel does not serve runs in
+// k_selgat's select-only form (its register-resident cut holds at most 4096
+// keys) rather than k_select: a budget known before the selection, no
+// diagnostics.
+inline bool fast_select_ok(const StepParams& p) {
+  return !p.anchor && p.mode != 4 && !p.n_act && !p.act_bits && p.max_visual <= 4096;
+}
+inline int select_kind(const StepParams& p, int kept_cap) {
+  return fused_select_gather_ok(p, kept_cap) ? 1 : fast_select_ok(p) ? 2 : 0;
 }
 
 // Launch plan and copy descriptors of a decode step (p's shapes, inputs and

@@ -3292,10 +3292,29 @@ __device__ __forceinline__ RadixCut radix_cut_regs(const uint32_t (&k)[kCutKeys]
   return RadixCut{whole ? prefix - 1u : prefix, krem, n_theta, whole};
 }
 
+// Exclusive prefix sum over the block with one barrier: wsum_s[NTH / 32]
+// must not be written again before the next barrier.
+template <int NTH>
+__device__ __forceinline__ int block_excl_scan_1b(int x, int* wsum_s) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += n;
+  }
+  if (lane == 31) wsum_s[warp] = incl;
+  __syncthreads();
+  int before = 0;
+  for (int w = 0; w < warp; ++w) before += wsum_s[w];
+  return before + incl - x;
+}
+
 // Ascending compaction of the register-resident keys (see radix_cut_regs):
 // keys above c.theta plus the first c.krem keys equal to it (every key when
-// take_all), written to kept (global) and kept_s (shared memory).
-template <int NTH>
+// take_all), written to kept (global) and, with TO_SMEM, to kept_s (shared
+// memory).  wsum_s holds 2 * NTH / 32 ints.
+template <int NTH, bool TO_SMEM>
 __device__ __forceinline__ void compact_kept_regs(const uint32_t (&k)[kCutKeys], int nvalid, int K, bool take_all,
                                                   const RadixCut& c, int* wsum_s, int32_t* kept, int* kept_s) {
   const int i0 = kCutKeys * (int)threadIdx.x;
@@ -3304,7 +3323,7 @@ __device__ __forceinline__ void compact_kept_regs(const uint32_t (&k)[kCutKeys],
   if (ties)
 #pragma unroll
     for (int j = 0; j < kCutKeys; ++j) n_eq += j < nvalid && k[j] == c.theta;
-  const int eq_before = ties ? block_excl_scan(n_eq, wsum_s) : 0;
+  const int eq_before = ties ? block_excl_scan_1b<NTH>(n_eq, wsum_s + NTH / 32) : 0;
   const unsigned krem = ties ? c.krem : 0xffffffffu;
   unsigned selm = 0;
   {
@@ -3317,12 +3336,12 @@ __device__ __forceinline__ void compact_kept_regs(const uint32_t (&k)[kCutKeys],
       selm |= (unsigned)sel << j;
     }
   }
-  int o = block_excl_scan(__popc(selm), wsum_s);
+  int o = block_excl_scan_1b<NTH>(__popc(selm), wsum_s);
 #pragma unroll
   for (int j = 0; j < kCutKeys; ++j)
     if (((selm >> j) & 1u) && o < K) {
       kept[o] = i0 + j;
-      kept_s[o] = i0 + j;
+      if constexpr (TO_SMEM) kept_s[o] = i0 + j;
       ++o;
     }
 }
@@ -3351,7 +3370,10 @@ constexpr int kSgTextSplits = 10;  // text split partials a thread requests ahea
 // pieces XOR-swizzled by the row so that ldmatrix reads hit distinct banks.
 __device__ __forceinline__ unsigned sg_swz(int j, int c) { return (unsigned)(j * 128 + ((c ^ (j & 7)) << 4)); }
 
-template <typename T, int D, int GM>
+// GATHER = false: the selection alone (steps 1, 2b and 3), for calls whose
+// gather runs as its own kernel; it also writes every head's largest logit
+// (p.hmax) for that kernel.
+template <typename T, int D, int GM, bool GATHER = true>
 __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ StepParams p) {
   constexpr int NTH = kSgThreads, NW = kSgWarps;
   constexpr bool BF = sizeof(T) == 2;
@@ -3367,10 +3389,10 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   const int G = p.G, H = p.H, ns = p.ns, nv = sq.nv;
   // This CTA's output: kv-head g, dimensions [d0, d0 + W) (the plan makes
   // the cluster split every kv-head evenly, W a multiple of 16).
-  const int rpg = p.granularity ? ncl : ncl / p.Hkv;
-  const int W = D / rpg;
-  const int g = p.granularity ? gsel : rank / rpg;
-  const int d0 = (rank % rpg) * W;
+  const int rpg = !GATHER ? 1 : p.granularity ? ncl : ncl / p.Hkv;
+  const int W = GATHER ? D / rpg : 16;
+  const int g = !GATHER ? 0 : p.granularity ? gsel : rank / rpg;
+  const int d0 = GATHER ? (rank % rpg) * W : 0;
   const int64_t hrow0 = (int64_t)b * H + g * G;
   const int nsel = p.granularity ? p.Hkv : 1;
   pdl_wait();
@@ -3462,7 +3484,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
       sm.hInv[h] = L1 > 0.f ? 1.f / L1 : 0.f;
       sm.hMass[h] = Lta > 0.f ? Ltv / Lta : 0.f;
       sm.hMass1[h] = L1 > 0.f ? L1v / L1 : 0.f;
-      if (h >= g * G && h < g * G + G) { sm.hMt[h - g * G] = Mt; sm.hLt[h - g * G] = Lt; }
+      if (GATHER && h >= g * G && h < g * G + G) { sm.hMt[h - g * G] = Mt; sm.hLt[h - g * G] = Lt; }
     }
   }
   __syncthreads();
@@ -3479,12 +3501,14 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   const float* tso = p.split_o + (hrow0 + th) * p.nsp_max * D + tdim;
   float tmx[kSgTextSplits];
   float4 tov[kSgTextSplits];
+  if constexpr (GATHER) {
 #pragma unroll
-  for (int k = 0; k < kSgTextSplits; ++k) {
-    const int s = tsg + 4 * k;
-    const bool ok = tlive && s < ns;
-    tmx[k] = ok ? __ldcg(tst + (int64_t)s * ST_N) : -CUDART_INF_F;
-    tov[k] = ok ? __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k = 0; k < kSgTextSplits; ++k) {
+      const int s = tsg + 4 * k;
+      const bool ok = tlive && s < ns;
+      tmx[k] = ok ? __ldcg(tst + (int64_t)s * ST_N) : -CUDART_INF_F;
+      tov[k] = ok ? __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
 
   // Rank 0: head mean, head max (Sec. 4.3) and the budget (Eq. 7), on the
@@ -3501,7 +3525,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
       mx = warp_max(mx);
       s1 = warp_sum(s1);
       if (lane == 0) {
-        const int K = min(budget_k(p, mx, nv), min(p.kept_cap, kSliceMaxKept));
+        const int K = min(budget_k(p, mx, nv), GATHER ? min(p.kept_cap, kSliceMaxKept) : p.kept_cap);
         sm.K = K;
         p.kept_count[(int64_t)b * nsel + gsel] = K;
         if (gsel == 0 && p.mass_stats) {
@@ -3510,7 +3534,10 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
         }
       }
     } else if (gsel == 0) {
-      for (int h = tid; h < H; h += NTH - 32) p.mass[(int64_t)b * H + h] = sm.hMass[h];
+      for (int h = tid; h < H; h += NTH - 32) {
+        p.mass[(int64_t)b * H + h] = sm.hMass[h];
+        if constexpr (!GATHER) p.hmax[(int64_t)b * H + h] = sm.hM[h];
+      }
     }
   }
 
@@ -3554,7 +3581,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
 
   // 2c. The text part: sum exp2(m_s - m_text) * o_s over the splits, then over
   //     the element's four split groups.
-  {
+  if constexpr (GATHER) {
     const float tmh = sm.hMt[th];
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -3578,6 +3605,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   }
   if (ncl > 1) cluster.sync();  // rank 0 now sees every key
   else __syncthreads();
+  if (!GATHER && rank != 0) return;  // nothing reads this CTA's shared memory any more
 
   // 3. Rank 0: the Top-K_t cut (Eq. 3) and the ascending compaction, with
   //    every thread's eight keys in registers, into the output and into its
@@ -3597,9 +3625,10 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
     RadixCut cut{0u, (unsigned)K, 0u, false};
     __syncthreads();  // every key is in registers: the key array holds the warps' histograms from here on
     if (K > 0 && !take_all) cut = radix_cut_regs<NTH>(kr, nvalid, K, key_s, sm.tot);
-    if (K > 0) compact_kept_regs<NTH>(kr, nvalid, K, take_all, cut, sm.wsum, kept, sm.kept);
+    if (K > 0) compact_kept_regs<NTH, GATHER>(kr, nvalid, K, take_all, cut, sm.wsum, kept, sm.kept);
     for (int i = max(K, 0) + tid; i < p.kept_cap; i += NTH) kept[i] = -1;
   }
+  if constexpr (!GATHER) return;
   if (ncl > 1) cluster.sync();  // rank 0 holds the kept list
   else __syncthreads();
   // Every CTA copies the budget and the kept list from rank 0, then lets
@@ -3902,7 +3931,7 @@ cudaError_t launch_score(const StepParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_gather(const StepParams& p, cudaStream_t st) {
-  if (p.fused) return cudaSuccess;  // the select kernel gathered
+  if (p.fused == 1) return cudaSuccess;  // the select kernel gathered
   if (p.dtype == 0)
     return p.D == 128 ? launch_gather_td<__nv_bfloat16, 128>(p, st) : launch_gather_td<__nv_bfloat16, 64>(p, st);
   return p.D == 128 ? launch_gather_td<float, 128>(p, st) : launch_gather_td<float, 64>(p, st);
@@ -3940,7 +3969,10 @@ cudaError_t launch_selgat_td(const StepParams& p, dim3 grid, size_t smem, cudaSt
 
 cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
   const dim3 grid(p.cl, p.granularity ? p.Hkv : 1, p.B);
-  if (p.fused) {
+  if (p.fused == 2)
+    return launch_ex(k_selgat<__nv_bfloat16, 128, 8, false>, grid, dim3(kSgThreads),
+                     selgat_smem_bytes(p.max_visual, 0), st, p.cl, p);
+  if (p.fused == 1) {
     const size_t smem = selgat_smem_bytes(p.max_visual, p.dtype);
     if (p.dtype == 0)
       return p.D == 128 ? launch_selgat_td<__nv_bfloat16, 128>(p, grid, smem, st)
@@ -4055,6 +4087,12 @@ cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {
     cudaFuncAttributes attr;
     if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k);
     if (e == cudaSuccess && attr.maxDynamicSharedSizeBytes < need) e = set_smem(k, need);
+  }
+  {
+    cudaFuncAttributes attr;
+    const int need = (int)selgat_smem_bytes(max_visual, 0);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k_selgat<__nv_bfloat16, 128, 8, false>);
+    if (e == cudaSuccess && attr.maxDynamicSharedSizeBytes < need) e = set_smem(k_selgat<__nv_bfloat16, 128, 8, false>, need);
   }
   void (*const selgat[2][4])(StepParams) = {
       {k_selgat<__nv_bfloat16, 128, 4>, k_selgat<__nv_bfloat16, 128, 8>, k_selgat<__nv_bfloat16, 64, 4>,

@@ -209,7 +209,7 @@ extern "C" vp_status vp_decode_step_noalloc(const vp_config* cfg, int32_t batch,
   p.nk_max = L.nk_max;
   if (!vp::plan_step(p, slot->num_sms, kept_cap, budget->granularity))
     return fail(VP_ERR_UNSUPPORTED, "vp_decode_step_noalloc: no launch plan serves this call");
-  p.fused = vp::fused_select_gather_ok(p, kept_cap) ? 1 : 0;
+  p.fused = vp::select_kind(p, kept_cap);
 
   // Only now that every check has passed: clear the counters, then launch.
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
