@@ -143,3 +143,25 @@ def test_tc_refuses_what_it_cannot_serve(vp):
             assert ei.value.status == vp.VP_ERR_INVALID_ARG
         finally:
             dev.close()
+
+
+def test_tc_ragged_lengths_one_long_sequence(vp):
+    """Very different lengths in one call: one long sequence among short ones
+    (splits of the long one's size, empty splits for the short ones), an
+    empty visual span, one-token sequences, text before the span."""
+    r = small(batch=12, vis_len=(1000, 64, 300, 0, 577, 128, 900, 1, 33, 700, 256, 512),
+              vis_start=(0, 5, 40, 0, 13, 0, 7, 0, 2, 0, 0, 100),
+              text_len=(9000, 20, 300, 5, 70, 1500, 129, 1, 2, 40, 2500, 300), seed=33)
+    tc_check(vp, r)
+    tc_check(vp, r, budget=dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=200_000))
+
+
+def test_tc_paged_ragged_batch(vp):
+    """A paged batch with text lengths spread like batched serving's, on the
+    automatic path (which picks the tcgen05 kernel) and forced."""
+    rng = np.random.default_rng(34)
+    text = tuple(int(t) for t in rng.integers(50, 3000, 16))
+    r = small(batch=16, vis_len=640, vis_start=0, text_len=text, paged=True, page_size=16, seed=34)
+    inp = Hn.make_inputs(r)
+    tc_check(vp, r, inp=inp)
+    Hn.check_all(vp, inp, r.budget)
