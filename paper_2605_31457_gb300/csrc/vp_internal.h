@@ -98,6 +98,7 @@ struct StepParams {
   int fused;          // select kernel: 0 k_select; 1 k_selgat, which also gathers (fused_select_gather_ok);
                       // 2 k_selgat selecting only (fast_select_ok)
   int split_w;        // weight of one score split (bulk-tensor kernel)
+  int num_sms;        // SMs of the device (launch shapes chosen per call)
 };
 
 // ---------------------------------------------------------------- host planning
@@ -289,6 +290,7 @@ inline int select_kind(const StepParams& p, int kept_cap) {
 // path: 0 the choice above, 1 never the tensor-core kernel, 2 only it
 // (false when it cannot serve the call).
 inline bool plan_step(StepParams& p, int num_sms, int kept_cap, int granularity, int path = 0) {
+  p.num_sms = num_sms;
   const long long w_tc = 2LL * ((p.max_seq + kTcRows - 1) / kTcRows) - p.max_visual / kTcRows;
   const bool eligible = tc_eligible(p.dtype, p.D, p.G, p.paged, p.page_size);
   const bool tc = path == 2 ? eligible

@@ -2720,18 +2720,22 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // k_gather_mma (bf16): grid (nc, Hkv, B), 4 warps.  CTA c (a) attends over
 // chunk c of the kept list (c < nk).  Warp w takes 32-token tiles w, w + 4,
 // ... of the chunk and streams the kept V rows through a private ring of
-// S slots (three; one when no chunk holds more than a tile per warp, so that
-// the smaller shared-memory footprint lets four CTAs share an SM): lane t
-// bulk-copies row t of a tile into a row padded to 2D + 16 bytes
-// (conflict-free ldmatrix), after lane 0 armed the slot's mbarrier with the
-// tile's byte count.  The tile's logits (read one tile
-// ahead) give per-head running maxima and probabilities; P.V runs on the
-// tensor cores as in the score kernel (A = V^T by ldmatrix.trans, B = P^T
-// from a per-warp bf16 buffer).  The warps' partials are merged into the
-// chunk's partial; (b) and the final combine are shared with k_gather.
+// S slots: the lanes copy a tile's V rows in 16-byte pieces (cp.async) into
+// a 128-byte-swizzled slot (conflict-free ldmatrix), with the tile's logits,
+// and the slot's mbarrier completes once all 32 lanes' copies have landed.
+// The kept indices are read from the kept list one tile ahead of their
+// copies.  S is 1 when no chunk holds more than one tile per warp (four CTAs
+// share an SM); otherwise 3 (two CTAs per SM) or 2 (three CTAs per SM,
+// the same bytes in flight per SM over more warps), whichever runs the grid
+// in fewer waves, 3 on a tie (a lone CTA in a short last wave keeps more
+// copies in flight).  The tile's logits give per-head probabilities; P.V
+// runs on the tensor cores as in the score kernel (A = V^T by
+// ldmatrix.trans, B = P^T from a per-warp bf16 buffer).  The warps'
+// partials are merged into the chunk's partial; (b) and the final combine
+// are shared with k_gather.
 // ---------------------------------------------------------------------------
 constexpr int kGmWarps = 4;
-constexpr int kGmSlots = 3;
+constexpr int kGmSlots = 3;  // ring slots of the deeper form (the other has 2)
 
 template <int D, int NT, int S>
 struct GmCfg {
@@ -2756,8 +2760,7 @@ struct GmCfg {
   static constexpr int OFF_WST = OFF_MASK + kGmWarps * S * 4;           // float [warps][GM][2]
   static constexpr int OFF_FIN = OFF_WST + kGmWarps * GM * 2 * 4;       // float [GM][4]
   static constexpr int OFF_LAST = OFF_FIN + GM * 4 * 4;
-  static constexpr int OFF_KIDX = OFF_LAST + 16;                // int16 [MAX_CHUNK] kept indices
-  static constexpr size_t SMEM = (size_t)OFF_KIDX + MAX_CHUNK * 2;
+  static constexpr size_t SMEM = (size_t)OFF_LAST + 16;
   static_assert(OFF_BAR % 8 == 0 && OFF_Z % 16 == 0 && OFF_WST % 16 == 0, "alignment");
 };
 
@@ -2776,7 +2779,6 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   float (*wst)[GM][2] = reinterpret_cast<float (*)[GM][2]>(smem + C::OFF_WST);
   float (*fin)[4] = reinterpret_cast<float (*)[4]>(smem + C::OFF_FIN);
   int* last = reinterpret_cast<int*>(smem + C::OFF_LAST);
-  short* kidx = reinterpret_cast<short*>(smem + C::OFF_KIDX);  // indices < 32768
   unsigned char* ring = smem + warp * S * C::SLOT;
 
   // A slot's phase completes when all 32 lanes' copies have landed.
@@ -2815,22 +2817,22 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
     const int per = (K + p.nk - 1) / p.nk;
     const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + C::MAX_CHUNK));
     if (per > C::MAX_CHUNK) err |= ERR_KEPT;  // the plan keeps every chunk within the limit
-    // The chunk's kept indices, read once (out-of-range ones become -1).
-    for (int j = j0 + tid; j < j1; j += C::THREADS) {
-      int i = __ldg(kept + j);
-      if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
-      kidx[j - j0] = (short)i;
-    }
     const int ntile = (j1 - j0 + 31) / 32;
     const int nj = warp < ntile ? (ntile - warp + kGmWarps - 1) / kGmWarps : 0;  // this warp's tiles
     const float* zb = p.z_ws + (int64_t)b * p.max_visual * p.hp + g * G;
     int issued = 0;  // tiles of this warp whose copies were issued
-    __syncthreads();
 
-    // Kept index of row `lane` of this warp's tile k, or -1.
+    // Kept index of row `lane` of this warp's tile k, or -1 (read from the
+    // kept list a tile ahead of its copies; an out-of-range index is
+    // flagged and skipped).
     auto row_index = [&](int k) {
       const int j = 32 * (warp + kGmWarps * k) + lane;
-      return (k < nj && j0 + j < j1) ? (int)kidx[j] : -1;
+      int i = -1;
+      if (k < nj && j0 + j < j1) {
+        i = __ldg(kept + j0 + j);
+        if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
+      }
+      return i;
     };
     auto issue = [&](int k, int i) {  // all lanes; i = this lane's kept index
       if (k >= nj) return;
@@ -3833,6 +3835,27 @@ cudaError_t launch_score_d(const StepParams& p, cudaStream_t st) {
 template <int GM>
 size_t slice_smem() { return sizeof(SliceSmem<GM>); }
 
+// CTAs of a chunk-gather instance resident on one SM (queried once).
+template <int D, int NT, int S>
+int gm_blocks_per_sm() {
+  static const int n = [] {
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, k_gather_mma<D, NT, S>, 32 * kGmWarps,
+                                                      GmCfg<D, NT, S>::SMEM) != cudaSuccess)
+      b = 0;
+    return b;
+  }();
+  return n;
+}
+// True when the two-slot form runs n CTAs in fewer waves than the three-slot one.
+template <int D, int NT>
+bool gm_fewer_waves(long long n, int num_sms) {
+  const long long r2 = (long long)gm_blocks_per_sm<D, NT, 2>() * num_sms;
+  const long long r3 = (long long)gm_blocks_per_sm<D, NT, kGmSlots>() * num_sms;
+  if (r2 <= 0 || r3 <= 0) return false;
+  return (n + r2 - 1) / r2 < (n + r3 - 1) / r3;
+}
+
 template <typename T, int D>
 cudaError_t launch_gather_td(const StepParams& p, cudaStream_t st) {
   if (p.gslice) {
@@ -3846,11 +3869,16 @@ cudaError_t launch_gather_td(const StepParams& p, cudaStream_t st) {
     // A single ring slot when no chunk can hold more than one tile per warp.
     const int kmax = min(p.kept_cap, p.max_visual);
     const bool one = p.nk == 0 || (kmax + p.nk - 1) / p.nk <= GmCfg<D, 1, 1>::MAX_CHUNK;
+    const long long n = (long long)p.nc * p.Hkv * p.B;
     if (p.G <= 8) {
       if (one) return launch_ex(k_gather_mma<D, 1, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 1, 1>::SMEM, st, 1, p);
+      if (gm_fewer_waves<D, 1>(n, p.num_sms))
+        return launch_ex(k_gather_mma<D, 1, 2>, grid, dim3(32 * kGmWarps), GmCfg<D, 1, 2>::SMEM, st, 1, p);
       return launch_ex(k_gather_mma<D, 1, kGmSlots>, grid, dim3(32 * kGmWarps), GmCfg<D, 1, kGmSlots>::SMEM, st, 1, p);
     }
     if (one) return launch_ex(k_gather_mma<D, 2, 1>, grid, dim3(32 * kGmWarps), GmCfg<D, 2, 1>::SMEM, st, 1, p);
+    if (gm_fewer_waves<D, 2>(n, p.num_sms))
+      return launch_ex(k_gather_mma<D, 2, 2>, grid, dim3(32 * kGmWarps), GmCfg<D, 2, 2>::SMEM, st, 1, p);
     return launch_ex(k_gather_mma<D, 2, kGmSlots>, grid, dim3(32 * kGmWarps), GmCfg<D, 2, kGmSlots>::SMEM, st, 1, p);
   }
   if (p.G <= 4) return launch_ex(k_gather<T, D, 4>, grid, dim3(kGatherThreads), gather_smem<T, D, 4>(), st, 1, p);
@@ -3872,6 +3900,10 @@ cudaError_t configure_fixed_kernels() {
   VP_SET((k_gather_mma<128, 2, kGmSlots>), (GmCfg<128, 2, kGmSlots>::SMEM));
   VP_SET((k_gather_mma<64, 1, kGmSlots>), (GmCfg<64, 1, kGmSlots>::SMEM));
   VP_SET((k_gather_mma<64, 2, kGmSlots>), (GmCfg<64, 2, kGmSlots>::SMEM));
+  VP_SET((k_gather_mma<128, 1, 2>), (GmCfg<128, 1, 2>::SMEM));
+  VP_SET((k_gather_mma<128, 2, 2>), (GmCfg<128, 2, 2>::SMEM));
+  VP_SET((k_gather_mma<64, 1, 2>), (GmCfg<64, 1, 2>::SMEM));
+  VP_SET((k_gather_mma<64, 2, 2>), (GmCfg<64, 2, 2>::SMEM));
   VP_SET((k_gather_mma<128, 1, 1>), (GmCfg<128, 1, 1>::SMEM));
   VP_SET((k_gather_mma<128, 2, 1>), (GmCfg<128, 2, 1>::SMEM));
   VP_SET((k_gather_mma<64, 1, 1>), (GmCfg<64, 1, 1>::SMEM));
@@ -3919,6 +3951,12 @@ cudaError_t configure_fixed_kernels() {
   VP_SET((k_gather_slice<float, 64, 8>), (slice_smem<8>()));
   VP_SET((k_gather_slice<float, 64, 16>), (slice_smem<16>()));
 #undef VP_SET
+  if (e == cudaSuccess) {  // the chunk gather's occupancies, now that its shared memory is set
+    gm_blocks_per_sm<128, 1, 2>(); gm_blocks_per_sm<128, 1, kGmSlots>();
+    gm_blocks_per_sm<128, 2, 2>(); gm_blocks_per_sm<128, 2, kGmSlots>();
+    gm_blocks_per_sm<64, 1, 2>(); gm_blocks_per_sm<64, 1, kGmSlots>();
+    gm_blocks_per_sm<64, 2, 2>(); gm_blocks_per_sm<64, 2, kGmSlots>();
+  }
   return e;
 }
 
