@@ -1262,9 +1262,9 @@ __device__ __forceinline__ int wg_sync_count(bool pred) {
 }
 
 // The 128-row tiles of one split.  Tiles [v0, v1) lie wholly inside the
-// visual span (K only, weight 1); every other tile carries text or padding
-// rows (K and V, weight 2).  Split s owns tiles [u0, u0 + n), a fixed weight
-// per split as in tma_split.
+// visual span (K only, weight kTcWv); every other tile carries text or
+// padding rows (K and V, weight kTcWt).  Split s owns tiles [u0, u0 + n), a
+// fixed weight per split as in tma_split.
 struct TcRange {
   int u0, n, v0, v1;
   __device__ __forceinline__ bool pure(int i) const { return u0 + i >= v0 && u0 + i < v1; }
@@ -1275,12 +1275,13 @@ __device__ __forceinline__ TcRange tc_split(const Seq& sq, int s, int ns, int sp
   TcRange r;
   r.v0 = (sq.vs + kTcRows - 1) / kTcRows;
   r.v1 = max(r.v0, min(NTl, (sq.vs + sq.nv) / kTcRows));
-  const int W = 2 * NTl - (r.v1 - r.v0);
+  const int W = kTcWt * NTl - (kTcWt - kTcWv) * (r.v1 - r.v0);
   const int per = max(split_w, (W + ns - 1) / ns);
+  const int wa = kTcWt * r.v0, wc = wa + kTcWv * (r.v1 - r.v0);  // weight before and up to the end of the span's tiles
   auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
-    if (w <= 2 * r.v0) return (w + 1) / 2;
-    if (w <= r.v0 + r.v1) return w - r.v0;
-    return (w + (r.v1 - r.v0) + 1) / 2;
+    if (w <= wa) return (w + kTcWt - 1) / kTcWt;
+    if (w <= wc) return r.v0 + (w - wa + kTcWv - 1) / kTcWv;
+    return r.v1 + (w - wc + kTcWt - 1) / kTcWt;
   };
   r.u0 = tile_of(min(W, s * per));
   r.n = tile_of(min(W, (s + 1) * per)) - r.u0;
@@ -1350,6 +1351,64 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
       vpg[i] = (pos < T && !tr.pure(t)) ? tma_page(p.v, p, b, pos) : -2;
     }
   }
+  // ---------------------------------------------------------------- copies
+  // Warp 0 issues the pieces in the order the tensor cores read them: K of
+  // tile i, then V of the text tile before it (its P.V follows tile i's QK);
+  // iteration n issues only the last V.  Lane 0 arms the slot's barrier;
+  // lane 2x + hh copies half hh of box x.
+  int qc = 0;              // pieces issued
+  int pi = 0, ppend = -1;  // next iteration; text tile whose V is due
+  auto issue = [&](int i, int part) {
+    const int sl = qc % S;
+    if (!__all_sync(0xffffffffu, mbar_wait(empty + sl, ((qc / S) & 1) ^ 1))) return false;
+    const int u = tr.u0 + i;
+    const int* pg = part ? vpg : kpg;
+    bool live = false, bad = false;
+    int base = b, row = 0;
+    const int x = lane >> 1, hh = lane & 1;
+    if (x < nb) {
+      const int pos = u * kTcRows + x * R;
+      if (pos < T) {
+        if (p.paged) {
+          base = pg[i * nb + x];
+          bad = base < 0;
+          row = pos & (p.page_size - 1);
+        } else {
+          row = pos;
+        }
+        live = !bad;
+      }
+    }
+    if (bad) err |= ERR_PAGE;
+    const unsigned n_live = __popc(__ballot_sync(0xffffffffu, live));  // live halves
+    if (lane == 0) mbar_expect_tx(full + sl, n_live * (unsigned)R * 128u);
+    __syncwarp();
+    if (live) {
+      auto crd = [&](int axis) { return axis == p.tpos ? row : axis == p.gpos ? g : base; };
+      tma_load_4d(smem_u32(smem + sl * C::SLOT) + hh * C::HALF + x * R * 128, part ? &p.tmv2 : &p.tmk2, 64 * hh,
+                  crd(1), crd(2), crd(3), full + sl);
+    }
+    ++qc;
+    return true;
+  };
+  // false when a wait gave up; with ring_only it stops before the first
+  // piece that would wait for a slot to be read.
+  auto produce = [&](bool ring_only) {
+    for (; pi <= n; ++pi) {
+      if (ring_only && qc + (pi < n ? 1 : 0) + (ppend >= 0 ? 1 : 0) > S) return true;
+      if (pi < n && !issue(pi, 0)) return false;
+      if (ppend >= 0 && !issue(ppend, 1)) return false;
+      ppend = (pi < n && !tr.pure(pi)) ? pi : -1;
+    }
+    return true;
+  };
+  bool timed_out = false;
+  // Contiguous caches: the first slots' copies start before the CTA-wide
+  // barrier; they need only the barriers that lane 0 initialised.
+  if (warp == 0 && !p.paged) {
+    __syncwarp();
+    timed_out = !produce(true);
+  }
   if (warp >= 2) {  // q of the kv-head's query heads, rows past G zero, K-major and swizzled
     const uint32_t* qb = reinterpret_cast<const uint32_t*>(reinterpret_cast<const __nv_bfloat16*>(p.q) +
                                                            ((int64_t)b * H + g * G) * D);
@@ -1368,58 +1427,12 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
   __syncthreads();
   tc_fence_after();
   const unsigned tmem = *tmem_slot;  // columns [0,16) and [16,32): S buffers; [32,48): O
-  bool timed_out = false;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ copies
-    // Pieces in the order the tensor cores read them: K of tile i, then V of
-    // the text tile before it (its P.V follows tile i's QK).  Lane 0 arms the
-    // slot's barrier; lane 2x + hh copies half hh of box x.
-    int q = 0;  // pieces issued
-    auto issue = [&](int i, int part) {
-      const int sl = q % S;
-      if (!__all_sync(0xffffffffu, mbar_wait(empty + sl, ((q / S) & 1) ^ 1))) return false;
-      const int u = tr.u0 + i;
-      const int* pg = part ? vpg : kpg;
-      bool live = false, bad = false;
-      int base = b, row = 0;
-      const int x = lane >> 1, hh = lane & 1;
-      if (x < nb) {
-        const int pos = u * kTcRows + x * R;
-        if (pos < T) {
-          if (p.paged) {
-            base = pg[i * nb + x];
-            bad = base < 0;
-            row = pos & (p.page_size - 1);
-          } else {
-            row = pos;
-          }
-          live = !bad;
-        }
-      }
-      if (bad) err |= ERR_PAGE;
-      const unsigned n_live = __popc(__ballot_sync(0xffffffffu, live));  // live halves
-      if (lane == 0) mbar_expect_tx(full + sl, n_live * (unsigned)R * 128u);
-      __syncwarp();
-      if (live) {
-        auto crd = [&](int axis) { return axis == p.tpos ? row : axis == p.gpos ? g : base; };
-        tma_load_4d(smem_u32(smem + sl * C::SLOT) + hh * C::HALF + x * R * 128, part ? &p.tmv2 : &p.tmk2, 64 * hh,
-                    crd(1), crd(2), crd(3), full + sl);
-      }
-      ++q;
-      return true;
-    };
-    {
-      int pend = -1;
-      for (int i = 0; i < n && !timed_out; ++i) {
-        if (!issue(i, 0) || (pend >= 0 && !issue(pend, 1))) { timed_out = true; break; }
-        pend = tr.pure(i) ? -1 : i;
-      }
-      if (!timed_out && pend >= 0 && !issue(pend, 1)) timed_out = true;
-      // Copies still in flight (only after a timeout can any be unread) land
-      // before the CTA's shared memory is released.
-      for (int k = max(0, q - S); k < q; ++k) mbar_wait(full + k % S, (k / S) & 1);
-    }
+    if (!timed_out && !produce(false)) timed_out = true;
+    // Copies still in flight (only after a timeout can any be unread) land
+    // before the CTA's shared memory is released.
+    for (int k = max(0, qc - S); k < qc; ++k) mbar_wait(full + k % S, (k / S) & 1);
   } else if (warp == 1) {
     // ------------------------------------------------------ tensor cores
     // Tile i's QK is issued before the P.V of the previous text tile, so that
@@ -1465,33 +1478,32 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
       pend = -1;
       return true;
     };
-    for (int i = 0; i < n; ++i) {
-      const int sb = i & 1, sk = q % S;
-      if (!wait_all(full + sk, (q / S) & 1) || !wait_all(s_free + sb, ((i >> 1) & 1) ^ 1)) {
-        timed_out = true;
-        break;
-      }
-      tc_fence_after();
-      if (lane == 0) {
-        const unsigned kb = smem_u32(smem + sk * C::SLOT), qs = smem_u32(smem + C::OFF_Q);
+    // Iteration n only multiplies the last text tile's P.V.
+    for (int i = 0; i <= n; ++i) {
+      if (i < n) {
+        const int sb = i & 1, sk = q % S;
+        if (!wait_all(full + sk, (q / S) & 1) || !wait_all(s_free + sb, ((i >> 1) & 1) ^ 1)) {
+          timed_out = true;
+          break;
+        }
+        tc_fence_after();
+        if (lane == 0) {
+          const unsigned kb = smem_u32(smem + sk * C::SLOT), qs = smem_u32(smem + C::OFF_Q);
 #pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks)
-          umma(tmem + 16 * sb, umma_desc(kb + (ks >> 2) * C::HALF + (ks & 3) * 32, 16, 1024),
-               umma_desc(qs + (ks >> 2) * C::QHALF + (ks & 3) * 32, 16, 1024), kIdQK, ks > 0);
-        umma_commit(s_full + sb);
-        umma_commit(empty + sk);
+          for (int ks = 0; ks < D / 16; ++ks)
+            umma(tmem + 16 * sb, umma_desc(kb + (ks >> 2) * C::HALF + (ks & 3) * 32, 16, 1024),
+                 umma_desc(qs + (ks >> 2) * C::QHALF + (ks & 3) * 32, 16, 1024), kIdQK, ks > 0);
+          umma_commit(s_full + sb);
+          umma_commit(empty + sk);
+        }
+        __syncwarp();
+        ++q;
       }
-      __syncwarp();
-      ++q;
       if (pend >= 0) {
         pq = q++;
         if (!pv()) { timed_out = true; break; }
       }
-      if (!tr.pure(i)) pend = i;
-    }
-    if (!timed_out && pend >= 0) {
-      pq = q++;
-      if (!pv()) timed_out = true;
+      if (i < n && !tr.pure(i)) pend = i;
     }
     if (lane == 0) umma_commit(mma_done);  // after every operation issued above
     __syncwarp();
@@ -4096,9 +4108,9 @@ void encode_kv_maps(StepParams& p) {
   p.tpos = kt; p.gpos = kg; p.bpos = kb;
   if (want_tc && tc_eligible(p.dtype, p.D, p.G, p.paged, p.page_size)) {
     // Page ids of a split's boxes are staged in shared memory: bound them
-    // (a split holds at most split_w + 1 tiles).
+    // (a split holds at most split_w / kTcWv + 1 tiles).
     const int R2 = p.paged ? (p.page_size < kTcRows ? p.page_size : kTcRows) : kTcRows;
-    const int64_t boxes = p.paged ? (int64_t)(p.split_w + 1) * (kTcRows / R2) : 0;
+    const int64_t boxes = p.paged ? (int64_t)(p.split_w / kTcWv + 1) * (kTcRows / R2) : 0;
     if (boxes <= kTcMaxBoxes && encode_one(p.k, p, &p.tmk2, &kt, &kg, &kb, R2) &&
         encode_one(p.v, p, &p.tmv2, &vt, &vg, &vb, R2) && kt == p.tpos && vt == p.tpos && kg == p.gpos &&
         vg == p.gpos && kb == p.bpos && vb == p.bpos)

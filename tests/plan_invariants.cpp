@@ -46,7 +46,8 @@ int main() {
                     const Plan pl = make_plan(B, Hkv, D, sms, mv, ms, cap, gran, tc != 0);
                     ++plans;
                     const long long TR = tc ? kTcRows : 32;
-                    long long w_max = 2LL * ((ms + TR - 1) / TR) - mv / TR;
+                    long long w_max = tc ? (long long)kTcWt * ((ms + TR - 1) / TR) - (long long)(kTcWt - kTcWv) * (mv / TR)
+                                         : 2LL * ((ms + TR - 1) / TR) - mv / TR;
                     if (w_max < 1) w_max = 1;
 #define CHECK(cond) check((cond), #cond, B, Hkv, D, sms, mv, ms, cap, tc, gran)
                     CHECK(pl.ns >= 1 && pl.ns <= kNsMax);
