@@ -2939,6 +2939,16 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
         // columns of heads past G hold stale bytes too; those heads' sums
         // are never read.)
         const uint32_t rb = mask >> (16 * sb);
+        if ((rb & 0xffffu) == 0xffffu) {  // all 16 rows copied (warp-uniform)
+#pragma unroll
+          for (int mi = 0; mi < C::MT; ++mi) {
+            uint32_t a0, a1, a2, a3;
+            ldsm_x4_t(vt + swz_off<C::HALF_BYTES>(16 * sb + vrow, 16 * mi + vcol), a0, a1, a2, a3);
+#pragma unroll
+            for (int nn = 0; nn < NT; ++nn) mma_bf16(acc[nn][mi], a0, a1, a2, a3, pb[nn][0], pb[nn][1]);
+          }
+          continue;
+        }
         const uint32_t mlo = (((rb >> (2 * tg)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 1)) & 1u) ? 0xffff0000u : 0u);
         const uint32_t mhi = (((rb >> (2 * tg + 8)) & 1u) ? 0x0000ffffu : 0u) | (((rb >> (2 * tg + 9)) & 1u) ? 0xffff0000u : 0u);
 #pragma unroll
