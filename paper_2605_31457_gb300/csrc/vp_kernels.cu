@@ -956,7 +956,10 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   const float ctau = p.inv_tau;
   bool timed_out = false;
   int qc = 0;  // first slot of the tile being read
-  if (!ANCHOR) pdl_wait();  // from here on the workspace is written
+  // The workspace (logits, partials) may still be read by the previous
+  // kernel: each thread waits for it only before its first workspace write,
+  // so splits of text tiles stream their whole range meanwhile.
+  bool ws_ok = ANCHOR;
 
   for (int j = 0; j < nj; ++j) {
     const int t = warp + NW * j;
@@ -997,6 +1000,11 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
     // c[sb][n][e]: row 16sb + gr + 8(e >> 1), head 8n + 2tg + (e & 1).
     float zv[2][NT][4], zt[2][NT][4];
     bool any_vis = false;
+    // A tile with visual rows writes logits: wait for the workspace first (warp-uniform).
+    if (!ws_ok && !kept_tile && p0 < sq.vs + sq.nv && p0 + kTmaTile > sq.vs) {
+      pdl_wait();
+      ws_ok = true;
+    }
 #pragma unroll
     for (int sb = 0; sb < 2; ++sb)
 #pragma unroll
@@ -1151,6 +1159,7 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
     }
   if (timed_out) err |= ERR_TIMEOUT;
   if (err) atomicOr(p.err, err);
+  if (!ws_ok) pdl_wait();
   score_epilogue<GM, D, NW, C::THREADS>(p, b, g, s, wst, reinterpret_cast<const float*>(smem), GM * D, tail);
 }
 
@@ -1523,7 +1532,11 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
     float* zbase = p.z_ws + (int64_t)b * p.max_visual * p.hp + g * G;
     const bool zvec = (G & 3) == 0;
     bool dead = false;  // a wait of this thread gave up: skip the work, keep the barriers
-    pdl_wait();         // from here on the workspace is written
+    // The workspace may still be read by the previous kernel: a thread waits
+    // for it only before its first workspace write (visual logits, or the
+    // split's partial), so splits of text tiles stream their whole range
+    // meanwhile.
+    bool ws_ok = false;
     int j = 0;          // text tiles seen
     for (int i = 0; i < n; ++i) {
       const int u = tr.u0 + i, sb = i & 1;
@@ -1538,6 +1551,12 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
       }
       tc_fence_before();
       mbar_arrive(s_free + sb);
+      // A tile with visual rows writes logits: wait for the workspace first
+      // (the same decision for every softmax thread).
+      if (!ws_ok && u * kTcRows < sq.vs + sq.nv && u * kTcRows + kTcRows > sq.vs) {
+        pdl_wait();
+        ws_ok = true;
+      }
       const int pos = u * kTcRows + r;
       bool valid = !dead && pos < T;
       if (valid && p.paged) valid = kpg[i * nb + r / R] >= 0;
@@ -1654,6 +1673,7 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
       }
     }
     wg_sync();
+    if (!ws_ok) pdl_wait();
     const int64_t rec0 = ((int64_t)b * H + g * G) * p.nsp_max + s;  // split slot of head 0
     if (r < G) {
       const int h = r;
