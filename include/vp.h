@@ -144,6 +144,15 @@ vp_status vp_init(const vp_config* cfg, vp_ctx** out_ctx);
  *   mass_stats   float [batch][4] or NULL: { M_vis(tau), M_vis,max(tau),
  *                M_vis(tau = 1), (float)K_t }.
  *   cuda_stream  cudaStream_t to enqueue on (NULL = legacy default stream).
+ * Calls on one stream overlap: a call's kernels start while those of the
+ * previous call of this library on the same stream finish (programmatic
+ * dependent launch), and vp_decode_step reads q, the caches, spans, lengths
+ * and page table before it waits for that call (it waits before its first
+ * workspace write).  So no input of vp_decode_step may be written by the
+ * immediately preceding call of this library on the stream; any other kernel
+ * or copy in between removes the overlap.  vp_compact_kv's output caches are
+ * exempt (its kernel completes before the next call starts), and
+ * vp_decode_gather waits for the previous call before reading its kept set.
  */
 vp_status vp_decode_step(vp_ctx* ctx, int32_t batch, const void* q,
                          const vp_kv* k_cache, const vp_kv* v_cache,

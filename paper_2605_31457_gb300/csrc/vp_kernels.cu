@@ -794,7 +794,7 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
   const int32_t* kept_rows = nullptr;
   if (ANCHOR) {
     const int sel = p.granularity ? b * p.Hkv + g : b;
-    const int c = __ldg(p.kept_count + sel);
+    const int c = __ldcg(p.kept_count + sel);
     if (c < 0 || c > min(p.kept_cap, sq.nv)) err |= ERR_KEPT;
     n_kept = max(0, min(c, min(p.kept_cap, sq.nv)));
     kept_rows = p.kept_idx + (int64_t)sel * p.kept_cap;
@@ -840,7 +840,7 @@ __global__ void __launch_bounds__(32 * NW, 1) k_score_tma(const __grid_constant_
         // the warp copies K and V in 16-byte pieces, two rows per instruction,
         // into the swizzled layout of the tensor copies.
         const int r = (tr.u0 + t - tr.ntext) * kTmaTile + lane;
-        int i = r < n_kept ? __ldg(kept_rows + r) : -1;
+        int i = r < n_kept ? __ldcg(kept_rows + r) : -1;
         if (r < n_kept && (i < 0 || i >= sq.nv)) { err |= ERR_KEPT; i = -1; }
         const __nv_bfloat16* kr = nullptr;
         const __nv_bfloat16* vr = nullptr;
@@ -1723,8 +1723,10 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
 constexpr int kCompactRows = 128;  // destination rows per CTA
 
 __global__ void __launch_bounds__(256) k_compact(const __grid_constant__ CompactParams c) {
-  pdl_wait();  // kept_idx / kept_count may come from the previous kernel
-  pdl_trigger();
+  // kept_idx / kept_count may come from the previous kernel.  No early
+  // trigger: the next call may read the caches written here before its own
+  // wait, so it starts only once this grid has completed.
+  pdl_wait();
   const int g = blockIdx.y, b = blockIdx.z;
   int vs = __ldg(c.vis_start + b), nv = __ldg(c.vis_len + b), tl = __ldg(c.text_len + b);
   unsigned e = 0;
@@ -1732,7 +1734,7 @@ __global__ void __launch_bounds__(256) k_compact(const __grid_constant__ Compact
   if (tl < 1) { e |= ERR_TEXT; tl = 1; }
   if (nv + tl > c.max_seq) { e |= ERR_LEN; tl = max(1, c.max_seq - nv); }
   if (vs < 0 || vs > tl) { e |= ERR_SPAN; vs = min(max(vs, 0), tl); }
-  int K = __ldg(c.kept_count + b);
+  int K = __ldcg(c.kept_count + b);
   if (K < 0 || K > min(c.kept_cap, nv)) { e |= ERR_KEPT; K = max(0, min(K, min(c.kept_cap, nv))); }
   const int Tn = K + tl;  // rows of the compacted sequence
   const int ppr = c.D * c.esz / 16;  // 16-byte pieces per row
@@ -1746,7 +1748,7 @@ __global__ void __launch_bounds__(256) k_compact(const __grid_constant__ Compact
     if (t < vs) {
       pos = t;
     } else if (t < vs + K) {
-      const int i = __ldg(c.kept_idx + (int64_t)b * c.kept_cap + (t - vs));
+      const int i = __ldcg(c.kept_idx + (int64_t)b * c.kept_cap + (t - vs));
       pos = (i >= 0 && i < nv) ? vs + i : -1;
       if (pos < 0) e |= ERR_KEPT;
     } else {
@@ -2630,7 +2632,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
   if (c < p.nk) {
     const Seq sq = load_seq(p, b, false);
     const int sel = p.granularity ? b * p.Hkv + g : b;
-    const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
+    const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
     const int per = (K + p.nk - 1) / p.nk;
     const int j0 = min(K, c * per), j1 = min(K, j0 + per);
@@ -2844,7 +2846,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   if (c < p.nk) {
     const Seq sq = load_seq(p, b, false);
     const int sel = p.granularity ? b * p.Hkv + g : b;
-    const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
+    const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
     const int per = (K + p.nk - 1) / p.nk;
     const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + C::MAX_CHUNK));
@@ -2861,7 +2863,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       const int j = 32 * (warp + kGmWarps * k) + lane;
       int i = -1;
       if (k < nj && j0 + j < j1) {
-        i = __ldg(kept + j0 + j);
+        i = __ldcg(kept + j0 + j);
         if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
       }
       return i;
@@ -3115,7 +3117,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
   pdl_wait();
   pdl_trigger();
   const int sel = p.granularity ? b * p.Hkv + g : b;
-  const int K = max(0, min(__ldg(p.kept_count + sel), min(sq.nv, min(p.kept_cap, kSliceMaxKept))));
+  const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, min(p.kept_cap, kSliceMaxKept))));
   const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
   unsigned err = 0;
 
@@ -3126,7 +3128,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
 #pragma unroll
   for (int t = 0; t < TPT; ++t) {
     const int j = j0 + TSTRIDE * t;
-    idx[t] = j < K ? __ldg(kept + j) : -1;
+    idx[t] = j < K ? __ldcg(kept + j) : -1;
     if (j < K && (idx[t] < 0 || idx[t] >= sq.nv)) { err |= ERR_KEPT; idx[t] = -1; }
   }
   float vv[TPT][CH];
@@ -3439,8 +3441,13 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   const int d0 = GATHER ? (rank % rpg) * W : 0;
   const int64_t hrow0 = (int64_t)b * H + g * G;
   const int nsel = p.granularity ? p.Hkv : 1;
+  // Fused: the next kernel is the next call's score kernel, which reads only
+  // its inputs before its own wait, so it may start now.  Select only: the
+  // gather kernel reads the score partials before its wait, which this
+  // kernel's wait guarantees complete.
+  if constexpr (GATHER) pdl_trigger();
   pdl_wait();
-  pdl_trigger();
+  if constexpr (!GATHER) pdl_trigger();
   const float inv_tau = p.inv_tau;
 
   // 1. Split statistics -> per-head max, normalisers and masses (Eq. 5,
