@@ -169,3 +169,45 @@ def test_compact_argument_errors(vp):
             assert st == want, st
     finally:
         dev.close()
+
+
+def test_compaction_then_decode_on_one_stream(vp):
+    """vp_compact_kv followed at once by vp_decode_step over the compacted
+    caches, on one stream with no host synchronisation in between: the decode
+    step reads its caches before it waits for the previous kernel, so the
+    compaction must have completed by the time it starts.  The result must be
+    bit-identical to the same calls with a synchronisation between them."""
+    r = small(vis_len=(1500, 577, 64), text_len=(2500, 70, 129))  # a compaction of a few MB
+    inp = Hn.make_inputs(r)
+    q_last = Hn.make_inputs(r, step=1).q
+    dev = Hn.Device(vp, dataclasses.replace(inp, q=q_last), FASTV)
+    try:
+        dev.run()  # FastV's selection with the last prompt token
+        kept, count = dev.kept[:, 0, :].contiguous(), dev.count[:, 0].contiguous()
+        span_c = vp.span(dev.vs, count)  # the survivors form the new visual span
+        decode_q = inp.q.cuda()
+        bd = vp.make_budget(**r.budget)
+        cap = max(1, vp.vp_max_kept(bd, dev.cfg.max_visual))
+        results = []
+        for sync in (True, False):
+            dst = [torch.zeros_like(dev.k_t), torch.zeros_like(dev.v_t)]
+            for src, d in zip((dev.kc, dev.vc), dst):
+                vp.vp_compact_kv(dev.ctx, dev.B, src, vp.kv_contiguous(d), dev.span, dev.tl, kept, dev.kept_cap,
+                                 count)
+            if sync:
+                torch.cuda.synchronize()
+            out = torch.full_like(dev.out, float("nan"))
+            kept2 = torch.full((dev.B, cap), -7, dtype=torch.int32, device="cuda")
+            count2 = torch.full((dev.B,), -7, dtype=torch.int32, device="cuda")
+            mass = torch.empty_like(dev.mass)
+            stats = torch.empty_like(dev.stats)
+            vp.vp_decode_step(dev.ctx, dev.B, decode_q, vp.kv_contiguous(dst[0]), vp.kv_contiguous(dst[1]), span_c,
+                              dev.tl, bd, out, kept2, cap, count2, mass, stats)
+            vp.vp_check_errors(dev.ctx)
+            torch.cuda.synchronize()
+            results.append((_bits(out.cpu()), kept2.cpu().numpy(), count2.cpu().numpy()))
+    finally:
+        dev.close()
+    for a, b in zip(results[0], results[1]):
+        np.testing.assert_array_equal(a, b)
+    assert (results[0][2] > 0).all()
