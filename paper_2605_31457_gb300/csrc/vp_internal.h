@@ -115,6 +115,50 @@ constexpr int kTcRows = 128;  // rows of a tile of the tensor-core score kernel
 // peak, 10 : 18 0.83, 10 : 16 0.84, 10 : 14 0.85, 10 : 12 0.84.
 constexpr int kTcWv = 10, kTcWt = 14;
 constexpr int kTcMaxBoxes = 384;  // page ids per cache a tensor-core score CTA stages
+
+// The 128-row tiles of one split of the tensor-core score kernel, for a
+// sequence of vis_len visual tokens starting at vis_start and text_len text
+// tokens.  Tiles [v0, v1) lie wholly inside the visual span (K only, weight
+// kTcWv); every other tile carries text or padding rows (K and V, weight
+// kTcWt).  Split s owns tiles [u0, u0 + n): the tiles whose weight prefix
+// falls in [s * per, (s + 1) * per), per = max(split_w, ceil(W / ns)), so the
+// splits partition the sequence's tiles; tc_max_split_tiles bounds n.
+struct TcRange {
+  int u0, n, v0, v1;
+  __host__ __device__ bool pure(int i) const { return u0 + i >= v0 && u0 + i < v1; }
+};
+__host__ __device__ inline TcRange tc_split(int vis_start, int vis_len, int text_len, int s, int ns, int split_w) {
+  const int T = vis_len + text_len;
+  const int NTl = (T + kTcRows - 1) / kTcRows;
+  TcRange r;
+  r.v0 = (vis_start + kTcRows - 1) / kTcRows;
+  const int vend = (vis_start + vis_len) / kTcRows;
+  r.v1 = NTl < vend ? NTl : vend;
+  if (r.v1 < r.v0) r.v1 = r.v0;
+  const int W = kTcWt * NTl - (kTcWt - kTcWv) * (r.v1 - r.v0);
+  const int fair = (W + ns - 1) / ns;
+  const int per = split_w > fair ? split_w : fair;
+  const int wa = kTcWt * r.v0, wc = wa + kTcWv * (r.v1 - r.v0);  // weight before and up to the end of the span's tiles
+  auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
+    if (w <= wa) return (w + kTcWt - 1) / kTcWt;
+    if (w <= wc) return r.v0 + (w - wa + kTcWv - 1) / kTcWv;
+    return r.v1 + (w - wc + kTcWt - 1) / kTcWt;
+  };
+  const int w0 = s * per < W ? s * per : W, w1 = (s + 1) * per < W ? (s + 1) * per : W;
+  r.u0 = tile_of(w0);
+  r.n = tile_of(w1) - r.u0;
+  return r;
+}
+// The most tiles a tc_split split holds for any sequence of at most max_seq
+// tokens: per is largest for a sequence with no visual tile (every tile
+// weighs kTcWt), and a split's tiles weigh at least kTcWv each, plus one for
+// the tile its weight range starts inside.
+inline int tc_max_split_tiles(int max_seq, int ns, int split_w) {
+  const long long ntl = (max_seq + kTcRows - 1) / kTcRows;
+  const long long fair = (kTcWt * ntl + ns - 1) / ns;
+  const long long per = split_w > fair ? split_w : fair;
+  return (int)(per / kTcWv + 1);
+}
 constexpr int kNsMax = 256;   // score splits per (sequence, kv-head)
 constexpr int kMaxMerge = 8;  // gather CTAs merging slices of the text partials
 

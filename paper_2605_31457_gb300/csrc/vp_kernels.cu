@@ -1270,33 +1270,6 @@ __device__ __forceinline__ int wg_sync_count(bool pred) {
   return n;
 }
 
-// The 128-row tiles of one split.  Tiles [v0, v1) lie wholly inside the
-// visual span (K only, weight kTcWv); every other tile carries text or
-// padding rows (K and V, weight kTcWt).  Split s owns tiles [u0, u0 + n), a
-// fixed weight per split as in tma_split.
-struct TcRange {
-  int u0, n, v0, v1;
-  __device__ __forceinline__ bool pure(int i) const { return u0 + i >= v0 && u0 + i < v1; }
-};
-__device__ __forceinline__ TcRange tc_split(const Seq& sq, int s, int ns, int split_w) {
-  const int T = sq.nv + sq.tl;
-  const int NTl = (T + kTcRows - 1) / kTcRows;
-  TcRange r;
-  r.v0 = (sq.vs + kTcRows - 1) / kTcRows;
-  r.v1 = max(r.v0, min(NTl, (sq.vs + sq.nv) / kTcRows));
-  const int W = kTcWt * NTl - (kTcWt - kTcWv) * (r.v1 - r.v0);
-  const int per = max(split_w, (W + ns - 1) / ns);
-  const int wa = kTcWt * r.v0, wc = wa + kTcWv * (r.v1 - r.v0);  // weight before and up to the end of the span's tiles
-  auto tile_of = [&](int w) {  // first tile whose weight prefix reaches w
-    if (w <= wa) return (w + kTcWt - 1) / kTcWt;
-    if (w <= wc) return r.v0 + (w - wa + kTcWv - 1) / kTcWv;
-    return r.v1 + (w - wc + kTcWt - 1) / kTcWt;
-  };
-  r.u0 = tile_of(min(W, s * per));
-  r.n = tile_of(min(W, (s + 1) * per)) - r.u0;
-  return r;
-}
-
 template <int GM, int NS = kTcSlots>
 __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const __grid_constant__ StepParams p) {
   using C = TcCfgT<NS>;
@@ -1344,7 +1317,7 @@ __global__ void __launch_bounds__(kTcThreads, NS <= 3 ? 2 : 1) k_score_tc(const 
   const int G = p.G, H = p.H;
   const Seq sq = load_seq(p, b, s == 0 && g == 0);
   const int T = sq.nv + sq.tl;
-  const TcRange tr = tc_split(sq, s, p.ns, p.split_w);
+  const TcRange tr = tc_split(sq.vs, sq.nv, sq.tl, s, p.ns, p.split_w);
   const int R = p.paged ? min(kTcRows, p.page_size) : kTcRows;  // rows per copied box
   const int nb = kTcRows / R;
   int n = tr.n;
@@ -4144,10 +4117,9 @@ void encode_kv_maps(StepParams& p) {
   if (kt != vt || kg != vg || kb != vb) return;  // both caches must share an axis order
   p.tpos = kt; p.gpos = kg; p.bpos = kb;
   if (want_tc && tc_eligible(p.dtype, p.D, p.G, p.paged, p.page_size)) {
-    // Page ids of a split's boxes are staged in shared memory: bound them
-    // (a split holds at most split_w / kTcWv + 1 tiles).
+    // Page ids of a split's boxes are staged in shared memory: bound them.
     const int R2 = p.paged ? (p.page_size < kTcRows ? p.page_size : kTcRows) : kTcRows;
-    const int64_t boxes = p.paged ? (int64_t)(p.split_w / kTcWv + 1) * (kTcRows / R2) : 0;
+    const int64_t boxes = p.paged ? (int64_t)tc_max_split_tiles(p.max_seq, p.ns, p.split_w) * (kTcRows / R2) : 0;
     if (boxes <= kTcMaxBoxes && encode_one(p.k, p, &p.tmk2, &kt, &kg, &kb, R2) &&
         encode_one(p.v, p, &p.tmv2, &vt, &vg, &vb, R2) && kt == p.tpos && vt == p.tpos && kg == p.gpos &&
         vg == p.gpos && kb == p.bpos && vb == p.bpos)

@@ -61,6 +61,27 @@ int main() {
                     CHECK(pl.nc == (pl.nk > pl.nm ? pl.nk : pl.nm));
                     CHECK(!pl.gslice || cap <= kSliceMaxKept);
                     CHECK(pl.cl == 1 || pl.cl == 2 || pl.cl == 4 || pl.cl == 8);
+                    if (tc && cap == 0 && gran == 0) {
+                      // The tensor-core splits of sequences up to these shapes
+                      // partition every sequence's tiles, each split within
+                      // tc_max_split_tiles (the page-id staging bound).
+                      const int nvs[] = {0, 1, mv / 3, mv};
+                      for (int nv : nvs)
+                        for (int vs : {0, 13, 128, 1000})
+                          for (int tl : {1, 200, ms - nv}) {
+                            if (tl < vs || tl < 1 || nv + tl > ms) continue;
+                            const int NTl = (nv + tl + kTcRows - 1) / kTcRows;
+                            int next = 0, total = 0;
+                            for (int sp = 0; sp < pl.ns; ++sp) {
+                              const TcRange r = tc_split(vs, nv, tl, sp, pl.ns, pl.split_w);
+                              CHECK(r.n >= 0 && r.u0 == next);
+                              CHECK(r.n <= tc_max_split_tiles(ms, pl.ns, pl.split_w));
+                              next = r.u0 + r.n;
+                              total += r.n;
+                            }
+                            CHECK(total == NTl);
+                          }
+                    }
 #undef CHECK
                   }
             }
