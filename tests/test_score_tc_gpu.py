@@ -165,3 +165,52 @@ def test_tc_paged_ragged_batch(vp):
     inp = Hn.make_inputs(r)
     tc_check(vp, r, inp=inp)
     Hn.check_all(vp, inp, r.budget)
+
+
+@pytest.mark.parametrize("path", ["tc", "mma"])
+@pytest.mark.parametrize("budget", [W.ADAPTIVE_5PCT, dict(mode=O.FIXED_RATIO, tau=0.1, ratio_ppm=500_000)])
+def test_back_to_back_calls_on_one_stream(vp, path, budget):
+    """Four layer calls on one context and stream with no host
+    synchronisation.  Each call's score kernel starts while the previous
+    call's select (and gather) still run and waits only before its first
+    workspace write, so its text-only splits stream meanwhile.  Every output
+    must be bit-identical to the same call run alone.  The 5% budget takes the
+    fused select + gather, the 50% one the select and the chunk gather."""
+    r = small(vis_len=(1024, 577), vis_start=(0, 40), text_len=(4000, 2600), batch=2)
+    layers = range(4)
+    devs = [Hn.Device(vp, Hn.make_inputs(r, layer), budget) for layer in layers]
+    ctx = devs[0].ctx
+    vp.vp_set_score_path(ctx, vp.VP_SCORE_TC if path == "tc" else vp.VP_SCORE_MMA)
+
+    def call(d):
+        outs = dict(out=torch.full_like(d.out, float("nan")), kept=torch.full_like(d.kept, -7),
+                    count=torch.full_like(d.count, -7), mass=torch.full_like(d.mass, float("nan")),
+                    stats=torch.full_like(d.stats, float("nan")))
+        vp.vp_decode_step(ctx, d.B, d.q, d.kc, d.vc, d.span, d.tl, d.budget, outs["out"], outs["kept"], d.kept_cap,
+                          outs["count"], outs["mass"], outs["stats"])
+        return outs
+
+    def host(o):
+        return dict(out=o["out"].view(torch.int16).cpu().numpy(), kept=o["kept"].cpu().numpy(),
+                    count=o["count"].cpu().numpy(), mass=o["mass"].cpu().numpy(), stats=o["stats"].cpu().numpy())
+
+    try:
+        alone = []
+        for d in devs:
+            o = call(d)
+            vp.vp_check_errors(ctx)
+            torch.cuda.synchronize()
+            alone.append(host(o))
+        chained = [call(d) for d in devs]
+        vp.vp_check_errors(ctx)
+        torch.cuda.synchronize()
+        for layer, (want, o) in enumerate(zip(alone, chained)):
+            got = host(o)
+            for k in want:
+                np.testing.assert_array_equal(got[k], want[k], err_msg=f"layer {layer} {k}")
+        assert (alone[0]["count"] > 0).all()
+        if path == "tc":
+            assert vp.vp_last_launch(ctx)[0] == vp.VP_SCORE_TC
+    finally:
+        for d in devs:
+            d.close()
