@@ -301,23 +301,29 @@ inline bool tc_eligible(int dtype, int D, int G, int paged, int page_size) {
   return dtype == 0 && D == 128 && G >= 1 && G <= 16 && (!paged || page_size >= 8);
 }
 
-// Whether one kernel (select + slice gather) serves the call: the slice
-// gather would (few sequences, kept sets of at most kSliceMaxKept rows), the
-// budget is known before the selection (not top-p), no diagnostics are
-// asked for, at most 8 query heads share a kv-head, and the select cluster's
-// CTAs split the output dimensions of every kv-head evenly into slices of 16
-// to 64 dimensions, and the score keys of a sequence fit in the cut's
-// registers (eight per thread of 512: N_v <= 4096).
+// Whether one kernel (select + gather) serves the call: kept sets of at most
+// kSliceMaxKept rows, the budget known before the selection (not top-p), no
+// diagnostics, at most 8 query heads per kv-head, the select cluster's CTAs
+// splitting the output dimensions of every kv-head evenly into slices of 16
+// to 128 dimensions (64 with fp32 caches), and the score keys of a sequence
+// fitting in the cut's registers (eight per thread of 512: N_v <= 4096).
+// The select clusters (at most half as many CTAs as SMs) run in one wave.
+// Output dimensions of one CTA of the fused select + gather: the cluster's
+// ranks split into the kv-heads (one kept set per sequence) or take the
+// selection's kv-head (per-kv-head sets), each rank a slice of D; 0 if the
+// ranks do not divide evenly.
+inline int selgat_slice_dims(const StepParams& p) {
+  const int hunits = p.granularity ? 1 : p.Hkv;
+  if (p.cl % hunits) return 0;
+  const int rpg = p.cl / hunits;
+  return p.D % rpg ? 0 : p.D / rpg;
+}
 inline bool fused_select_gather_ok(const StepParams& p, int kept_cap) {
-  if (!p.gslice || p.anchor || p.mode == 4 || p.n_act || p.act_bits || p.G > 8 || kept_cap > kSliceMaxKept ||
+  if (p.anchor || p.mode == 4 || p.n_act || p.act_bits || p.G > 8 || kept_cap > kSliceMaxKept ||
       p.max_visual > 4096)
     return false;
-  const int hunits = p.granularity ? 1 : p.Hkv;
-  if (p.cl % hunits) return false;
-  const int rpg = p.cl / hunits;
-  if (p.D % rpg) return false;
-  const int W = p.D / rpg;
-  return W >= 16 && W <= 64;
+  const int W = selgat_slice_dims(p);
+  return W >= 16 && W <= (p.dtype == 0 ? 128 : 64);
 }
 
 // Whether the selection of a call the fused kernel does not serve runs in

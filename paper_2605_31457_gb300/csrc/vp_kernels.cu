@@ -3228,7 +3228,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather_slice(const __grid_co
 // ---------------------------------------------------------------------------
 constexpr int kSgThreads = 512;
 constexpr int kSgWarps = kSgThreads / 32;
-constexpr int kSgMaxW = 64;  // output dimensions of one CTA, at most
+constexpr int kSgMaxW = 128;  // output dimensions of one CTA, at most (64 with fp32 caches)
 
 // Register-resident Top-K cut of the fused kernel (Eq. 3) over n <= 8 * NTH
 // score keys: thread t holds keys [8t, 8t + 8), valid while below n.  Keys
@@ -3388,6 +3388,12 @@ constexpr int kSgTextSplits = 10;  // text split partials a thread requests ahea
 // Byte offset of 16-byte piece c of row j in a stage of 128-byte rows, the
 // pieces XOR-swizzled by the row so that ldmatrix reads hit distinct banks.
 __device__ __forceinline__ unsigned sg_swz(int j, int c) { return (unsigned)(j * 128 + ((c ^ (j & 7)) << 4)); }
+// 16-byte piece c of kept row j of a bf16 V stage: rows of up to 64
+// dimensions (128 bytes, swizzled) per half, the second 64 dimensions of a
+// row in a second half of kSliceMaxKept rows.
+__device__ __forceinline__ unsigned sg_voff(int j, int c) {
+  return (unsigned)((c >> 3) * (kSliceMaxKept * 128)) + sg_swz(j, c & 7);
+}
 
 // GATHER = false: the selection alone (steps 1, 2b and 3), for calls whose
 // gather runs as its own kernel; it also writes every head's largest logit
@@ -3517,8 +3523,10 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   //     now and summed after the importance pass: thread (element
   //     e = (head, 4 dimensions), split group sg of four) takes splits
   //     sg, sg + 4, ...
-  const int W4 = W / 4, NE = G * W4;  // NE <= 128: four threads per element
-  const int te = tid >> 2, tsg = tid & 3;
+  // Four threads per element when NE <= 128, else two (NE <= 256).
+  const int W4 = W / 4, NE = G * W4;
+  const int TSH = NE > NTH / 4 ? 1 : 2, TSG = 1 << TSH;
+  const int te = tid >> TSH, tsg = tid & (TSG - 1);
   const bool tlive = te < NE;
   const int th = tlive ? te / W4 : 0, tdim = d0 + 4 * (tlive ? te % W4 : 0);
   const float* tst = p.split_st + (hrow0 + th) * p.nsp_max * ST_N + ST_MT;
@@ -3528,7 +3536,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   if constexpr (GATHER) {
 #pragma unroll
     for (int k = 0; k < kSgTextSplits; ++k) {
-      const int s = tsg + 4 * k;
+      const int s = tsg + TSG * k;
       const bool ok = tlive && s < ns;
       tmx[k] = ok ? __ldcg(tst + (int64_t)s * ST_N) : -CUDART_INF_F;
       tov[k] = ok ? __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D)) : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -3613,13 +3621,12 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
       const float w = exp2_rel(tmx[k], tmh);
       a.x = fmaf(w, tov[k].x, a.x); a.y = fmaf(w, tov[k].y, a.y); a.z = fmaf(w, tov[k].z, a.z); a.w = fmaf(w, tov[k].w, a.w);
     }
-    for (int s = tsg + 4 * kSgTextSplits; tlive && s < ns; s += 4) {
+    for (int s = tsg + TSG * kSgTextSplits; tlive && s < ns; s += TSG) {
       const float w = exp2_rel(__ldcg(tst + (int64_t)s * ST_N), tmh);
       const float4 v = __ldcg(reinterpret_cast<const float4*>(tso + (int64_t)s * D));
       a.x = fmaf(w, v.x, a.x); a.y = fmaf(w, v.y, a.y); a.z = fmaf(w, v.z, a.z); a.w = fmaf(w, v.w, a.w);
     }
-#pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
+    for (int o = 1; o < TSG; o <<= 1) {
       a.x += __shfl_xor_sync(0xffffffffu, a.x, o);
       a.y += __shfl_xor_sync(0xffffffffu, a.y, o);
       a.z += __shfl_xor_sync(0xffffffffu, a.z, o);
@@ -3686,7 +3693,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
   asm volatile("cp.async.commit_group;\n" ::: "memory");
   for (int i = tid; i < (BF ? K16 : K) * CPR; i += NTH) {
     const int j = i / CPR, c = i % CPR;
-    const unsigned off = BF ? sg_swz(j, c) : (unsigned)((j * CPR + c) * 16);
+    const unsigned off = BF ? sg_voff(j, c) : (unsigned)((j * CPR + c) * 16);
     const T* vr = nullptr;
     if (j < K) {
       const int id = sm.kept[j];
@@ -3743,7 +3750,7 @@ __global__ void __launch_bounds__(kSgThreads) k_selgat(const __grid_constant__ S
       const uint32_t b1 = *reinterpret_cast<const uint32_t*>(pr + 8);
       const int col = 16 * mt + vcol;
       uint32_t a0, a1, a2, a3;
-      ldsm_x4_t(smem_u32(vst) + sg_swz(16 * ks + vrow, col >> 3), a0, a1, a2, a3);
+      ldsm_x4_t(smem_u32(vst) + sg_voff(16 * ks + vrow, col >> 3), a0, a1, a2, a3);
       mma_bf16(acc, a0, a1, a2, a3, b0, b1);
     }
     float* rw = sm.red[warp];
@@ -4011,11 +4018,11 @@ cudaError_t launch_compact(const CompactParams& c, cudaStream_t st) {
 }
 
 // Dynamic shared memory of k_selgat: the score keys, then the cut's per-warp
-// histograms, then the kept rows' V slices (bf16: rows of 128 bytes; fp32:
-// rows of up to 256 bytes).
-size_t selgat_smem_bytes(int max_visual, int dtype) {
+// histograms, then the kept rows' V slices of W dimensions (bf16: one or two
+// halves of rows of 128 bytes; fp32: packed rows).
+size_t selgat_smem_bytes(int max_visual, int dtype, int W = 64) {
   const size_t keys = select_smem_bytes(max_visual);
-  const size_t stage = (size_t)kSliceMaxKept * (dtype == 0 ? 128 : kSgMaxW * 4);
+  const size_t stage = (size_t)kSliceMaxKept * (dtype == 0 ? (W > 64 ? 256 : 128) : W * 4);
   const size_t hist = (size_t)2 * kSgWarps * 256 * 4;  // the cut's per-warp histograms
   size_t n = keys > stage ? keys : stage;
   return n > hist ? n : hist;
@@ -4033,7 +4040,7 @@ cudaError_t launch_select(const StepParams& p, cudaStream_t st) {
     return launch_ex(k_selgat<__nv_bfloat16, 128, 8, false>, grid, dim3(kSgThreads),
                      selgat_smem_bytes(p.max_visual, 0), st, p.cl, p);
   if (p.fused == 1) {
-    const size_t smem = selgat_smem_bytes(p.max_visual, p.dtype);
+    const size_t smem = selgat_smem_bytes(p.max_visual, p.dtype, selgat_slice_dims(p));
     if (p.dtype == 0)
       return p.D == 128 ? launch_selgat_td<__nv_bfloat16, 128>(p, grid, smem, st)
                         : launch_selgat_td<__nv_bfloat16, 64>(p, grid, smem, st);
@@ -4158,7 +4165,7 @@ cudaError_t configure_kernels(int max_visual, int H, int nsp_max) {
        k_selgat<__nv_bfloat16, 64, 8>},
       {k_selgat<float, 128, 4>, k_selgat<float, 128, 8>, k_selgat<float, 64, 4>, k_selgat<float, 64, 8>}};
   for (int dt = 0; dt < 2; ++dt) {
-    const int need_sg = (int)selgat_smem_bytes(max_visual, dt);
+    const int need_sg = (int)selgat_smem_bytes(max_visual, dt, dt == 0 ? kSgMaxW : 64);
     for (void (*k)(StepParams) : selgat[dt]) {
       cudaFuncAttributes attr;
       if (e == cudaSuccess) e = cudaFuncGetAttributes(&attr, k);

@@ -263,6 +263,30 @@ def test_qwen7b_full_size_layer(vp):
         Hn.check_all(vp, inp, W.ADAPTIVE_10PCT, report=rep)
 
 
+@pytest.mark.parametrize("paged", [False, True])
+def test_fused_select_gather_full_width_slices(vp, paged):
+    """A batch whose select clusters hold one CTA per kv-head: the fused
+    select + gather then attends over the kept rows for all 128 output
+    dimensions of a kv-head in one CTA (V staged as two swizzled 64-dimension
+    halves, two threads per text-partial element).  Ragged spans and lengths,
+    every sequence against the oracle."""
+    rng = np.random.default_rng(17)
+    B = 20
+    vis = tuple(int(x) for x in rng.integers(64, 700, size=B))
+    start = tuple(int(x) for x in rng.integers(0, 40, size=B))
+    text = tuple(int(x) + start[i] for i, x in enumerate(rng.integers(40, 900, size=B)))
+    r = small(batch=B, vis_len=vis, vis_start=start, text_len=text, seed=13, paged=paged, page_size=16)
+    inp = Hn.make_inputs(r)
+    dev = Hn.Device(vp, inp, r.budget)
+    try:
+        gpu = dev.run()
+        assert vp.vp_last_launch(dev.ctx)[1] == 2, "the fused select + gather should serve this batch"
+        for b in range(B):
+            Hn.compare_seq(inp, gpu, b, r.budget)
+    finally:
+        dev.close()
+
+
 def test_serving_paged_full_size_layer(vp):
     """Batched serving: B = 32, paged (page 16), 2304 visual, text 512..4096,
     visual mass spread over [0.01, 0.4]: every sequence against the oracle."""
