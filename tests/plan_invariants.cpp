@@ -1,8 +1,11 @@
-// Host-only check of the launch planner (make_plan, ws_layout): over a grid of
-// shapes, every plan covers the whole cache with its score splits, stays inside
-// the workspace the context allocated, keeps every gather chunk within the
-// chunk kernel's limit and picks the slice gather only for kept sets it holds.
-// Prints one line per violation and exits non-zero if there was any.
+// Host-only check of the launch planner (make_plan, ws_layout, tc_split,
+// select_kind): over a grid of shapes, every plan covers the whole cache with
+// its score splits, stays inside the workspace the context allocated, splits
+// every sequence's tiles for the tensor-core kernel within the page-id
+// staging bound, keeps every gather chunk within the chunk kernel's limit and
+// picks the slice gather only for kept sets it holds; a table of call shapes
+// gets its expected select form.  Prints one line per violation and exits
+// non-zero if there was any.
 #include <cstdio>
 
 #include "vp_internal.h"
@@ -19,6 +22,52 @@ void check(bool ok, const char* what, int B, int Hkv, int D, int sms, int mv, in
 }
 
 bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+
+// The select form (select_kind) the planner picks for a call shape on a
+// 152-SM device: 1 fused select + gather, 2 select only, 0 the
+// shared-memory select; and the fused kernel's slice width.
+struct FormCase {
+  const char* name;
+  int B, H, Hkv, D, max_visual, max_seq, kept_cap, gran, dtype, mode, diag;
+  int want_kind, want_w;
+};
+
+int check_forms() {
+  using namespace vp;
+  const FormCase cases[] = {
+      // name, B, H, Hkv, D, N_v, max_seq, kept_cap, gran, dtype, mode, diag, kind, W
+      {"B=1 decode (28/4, N_v 1296)", 1, 28, 4, 128, 1296, 4113, 64, 0, 0, 0, 0, 1, 64},
+      {"long reasoning (B=8, N_v 4096)", 8, 28, 4, 128, 4096, 21000, 204, 0, 0, 0, 0, 1, 64},
+      {"batched serving (B=32, N_v 2304)", 32, 28, 4, 128, 2304, 6500, 115, 0, 0, 0, 0, 1, 128},
+      {"sweep B=64, 32/8, N_v 2304, 5%", 64, 32, 8, 128, 2304, 3400, 115, 0, 0, 0, 0, 2, 0},
+      {"sweep B=64, N_v 6400 (keys beyond the register cut)", 64, 32, 8, 128, 6400, 7500, 320, 0, 0, 0, 0, 0, 0},
+      {"kept sets above 256 rows", 8, 28, 4, 128, 4096, 21000, 2048, 0, 0, 0, 0, 2, 0},
+      {"top-p budget", 1, 28, 4, 128, 1296, 4113, 1296, 0, 0, 4, 0, 0, 0},
+      {"diagnostics on", 1, 28, 4, 128, 1296, 4113, 64, 0, 0, 0, 1, 0, 0},
+      {"tiny fp32 (8/2, D 64)", 1, 8, 2, 64, 576, 720, 28, 0, 1, 0, 0, 1, 16},
+      {"fp32 caches, one CTA per kv-head (W 128 > 64)", 32, 28, 4, 128, 2304, 6500, 115, 0, 1, 0, 0, 2, 0},
+      {"per-kv-head sets, B=3", 3, 28, 4, 128, 577, 700, 28, 1, 0, 0, 0, 1, 16},
+      {"G = 16 (more than 8 heads per kv-head)", 2, 32, 2, 128, 1024, 3000, 51, 0, 0, 0, 0, 2, 0},
+  };
+  int bad = 0;
+  for (const FormCase& c : cases) {
+    StepParams p{};
+    p.B = c.B; p.H = c.H; p.Hkv = c.Hkv; p.G = c.H / c.Hkv; p.D = c.D;
+    p.max_visual = c.max_visual; p.max_seq = c.max_seq; p.granularity = c.gran; p.dtype = c.dtype;
+    p.mode = c.mode;
+    p.n_act = c.diag ? reinterpret_cast<int32_t*>(16) : nullptr;
+    const Plan pl = make_plan(c.B, c.Hkv, c.D, 152, c.max_visual, c.max_seq, c.kept_cap, c.gran, false);
+    p.cl = pl.cl; p.gslice = pl.gslice;
+    const int kind = select_kind(p, c.kept_cap);
+    const int w = kind == 1 ? selgat_slice_dims(p) : 0;
+    if (kind != c.want_kind || w != c.want_w) {
+      std::printf("FAIL select form of %s: kind %d (want %d), slice %d (want %d), cluster %d\n", c.name, kind,
+                  c.want_kind, w, c.want_w, pl.cl);
+      ++bad;
+    }
+  }
+  return bad;
+}
 
 }  // namespace
 
@@ -86,5 +135,6 @@ int main() {
                   }
             }
   std::printf("%lld plans, %d violations\n", plans, fails);
+  fails += check_forms();
   return fails ? 1 : 0;
 }
