@@ -2727,11 +2727,12 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // k_gather_mma (bf16): grid (nc, Hkv, B), 4 warps.  CTA c (a) attends over
 // chunk c of the kept list (c < nk).  Warp w takes 32-token tiles w, w + 4,
 // ... of the chunk and streams the kept V rows through a private ring of
-// S slots: the lanes copy a tile's V rows in 16-byte pieces (cp.async) into
-// a 128-byte-swizzled slot (conflict-free ldmatrix), with the tile's logits,
-// and the slot's mbarrier completes once all 32 lanes' copies have landed.
-// The kept indices are read from the kept list one tile ahead of their
-// copies.  S is 1 when no chunk holds more than one tile per warp (four CTAs
+// S slots: lane j copies row j of a tile with one bulk copy into a slot of
+// padded rows (a 16-byte shift per row: conflict-free ldmatrix), and the
+// token's logits with 4-byte cp.async (heads 0-3 into the row's pad bytes);
+// the slot's mbarrier completes once the row bytes and every lane's logits
+// have landed.  The kept indices are read from the kept list one tile ahead
+// of their copies.  S is 1 when no chunk holds more than one tile per warp (four CTAs
 // share an SM); otherwise 3 (two CTAs per SM) or 2 (three CTAs per SM,
 // the same bytes in flight per SM over more warps), whichever runs the grid
 // in fewer waves, 3 on a tie (a lone CTA in a short last wave keeps more
@@ -2749,8 +2750,11 @@ struct GmCfg {
   static constexpr int GM = 8 * NT;
   static constexpr int THREADS = 32 * kGmWarps;
   static constexpr int MT = D / 16;
-  static constexpr int HALF_BYTES = 32 * 128;                   // 32 rows x 64 dimensions
-  static constexpr int SLOT = (D / 64) * HALF_BYTES;            // 32 V rows, swizzled
+  // 32 V rows at a pitch of 2D + 16 bytes; the pad of row j holds token j's
+  // logits of heads 0-3, the other heads' logits sit in a separate array.
+  static constexpr int RP = 2 * D + 16;
+  static constexpr int SLOT = 32 * RP;
+  static constexpr int ZX = GM - 4;
   // Kept rows per CTA: a single slot serves one tile per warp.
   static constexpr int MAX_CHUNK = S == 1 ? 32 * kGmWarps : kGmMaxChunk;
   // After part (a) the ring holds the warps' outputs, then the split weights;
@@ -2760,15 +2764,15 @@ struct GmCfg {
   static constexpr int REUSE_BYTES = OFF_TW + 2 * GM * kNsMax * 4;
   static constexpr int RING = RING_BYTES > REUSE_BYTES ? RING_BYTES : REUSE_BYTES;
   static constexpr int OFF_BAR = RING;                          // full[warps][slots]
-  // Logits of a slot's tokens, float [GM][32]; once read, the tile's bf16
-  // probabilities [GM][32] take their place.
-  static constexpr int OFF_Z = OFF_BAR + kGmWarps * S * 8;
-  static constexpr int OFF_MASK = OFF_Z + kGmWarps * S * GM * 32 * 4;   // copied rows per slot
+  static constexpr int OFF_P = OFF_BAR + kGmWarps * S * 8;      // bf16 [warps][GM][32] probabilities
+  static constexpr int OFF_ZX = OFF_P + kGmWarps * GM * 32 * 2; // float [warps][slots][ZX][32] logits
+  static constexpr int OFF_MASK = OFF_ZX + kGmWarps * S * ZX * 32 * 4;  // copied rows per slot
   static constexpr int OFF_WST = OFF_MASK + kGmWarps * S * 4;           // float [warps][GM][2]
   static constexpr int OFF_FIN = OFF_WST + kGmWarps * GM * 2 * 4;       // float [GM][4]
   static constexpr int OFF_LAST = OFF_FIN + GM * 4 * 4;
   static constexpr size_t SMEM = (size_t)OFF_LAST + 16;
-  static_assert(OFF_BAR % 8 == 0 && OFF_Z % 16 == 0 && OFF_WST % 16 == 0, "alignment");
+  static_assert(RP % 16 == 0 && (RP / 16) % 8 == 1, "row pitch: 16-byte aligned rows, one bank group apart");
+  static_assert(OFF_BAR % 8 == 0 && OFF_P % 16 == 0 && OFF_ZX % 16 == 0 && OFF_WST % 16 == 0, "alignment");
 };
 
 template <int D, int NT, int S>
@@ -2781,15 +2785,17 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gr = lane >> 2, tg = lane & 3;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + warp * S;
-  float* zs = reinterpret_cast<float*>(smem + C::OFF_Z) + warp * S * GM * 32;
+  __nv_bfloat16* P = reinterpret_cast<__nv_bfloat16*>(smem + C::OFF_P) + warp * GM * 32;
+  float* zx = reinterpret_cast<float*>(smem + C::OFF_ZX) + warp * S * C::ZX * 32;
   uint32_t* mask_s = reinterpret_cast<uint32_t*>(smem + C::OFF_MASK) + warp * S;
   float (*wst)[GM][2] = reinterpret_cast<float (*)[GM][2]>(smem + C::OFF_WST);
   float (*fin)[4] = reinterpret_cast<float (*)[4]>(smem + C::OFF_FIN);
   int* last = reinterpret_cast<int*>(smem + C::OFF_LAST);
   unsigned char* ring = smem + warp * S * C::SLOT;
 
-  // A slot's phase completes when all 32 lanes' copies have landed.
-  if (tid < kGmWarps * S) mbar_init(reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + tid, 32);
+  // A slot's phase completes on lane 0's arrival (with the row bytes as its
+  // transaction count) once the rows and every lane's logits have landed.
+  if (tid < kGmWarps * S) mbar_init(reinterpret_cast<uint64_t*>(smem + C::OFF_BAR) + tid, 1);
   mbar_fence_init();
   __syncthreads();
   const int G = p.G, H = p.H;
@@ -2809,6 +2815,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   pdl_trigger();
   if (c < p.nm && p.anchor) {
     gather_text_slice<D, GM, C::THREADS>(p, c, hrow0, tw, tl);
+    fence_proxy_async();
     __syncthreads();
   }
   const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
@@ -2850,26 +2857,23 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
         if (!vr) { err |= ERR_PAGE; i = -1; }
       }
       const unsigned m = __ballot_sync(0xffffffffu, vr != nullptr);
-      if (lane == 0) mask_s[slot] = m;
+      unsigned char* row = ring + slot * C::SLOT + lane * C::RP;
+      // The slot was last read by this warp's ldmatrix and loads (generic
+      // proxy); its rows are next written by bulk copies (async proxy).
+      fence_proxy_async();
       __syncwarp();  // every lane is done reading this slot
-      // V rows: instruction j copies piece (lane % PPR) of row j * RPI + lane / PPR.
-      constexpr int PPR = 2 * D / 16, RPI = 32 / PPR;
-      const unsigned sbase = smem_u32(ring + slot * C::SLOT);
-      const unsigned long long src = reinterpret_cast<unsigned long long>(vr);
-#pragma unroll
-      for (int j = 0; j < 32 / RPI; ++j) {
-        const int row = j * RPI + lane / PPR;
-        const unsigned long long r = __shfl_sync(0xffffffffu, src, row);
-        if (r) cp_async16(sbase + swz_off<C::HALF_BYTES>(row, 8 * (lane % PPR)),
-                          reinterpret_cast<const char*>(r) + (lane % PPR) * 16);
-      }
-      // Logits of this lane's token.
+      if (lane == 0) mask_s[slot] = m;
+      // Logits of this lane's token: heads 0-3 into its row's pad.
       if (vr) {
         const float* zr = zb + (int64_t)i * p.hp;
-        const unsigned zd = smem_u32(zs + slot * GM * 32 + lane);
-        for (int h = 0; h < G; ++h) cp_async4(zd + h * 32 * 4, zr + h);
+        for (int h = 0; h < G; ++h)
+          cp_async4(h < 4 ? smem_u32(row + 2 * D + 4 * h) : smem_u32(zx + (slot * C::ZX + h - 4) * 32 + lane), zr + h);
       }
-      cp_async_arrive(full + slot);
+      cp_async_arrive_counted(full + slot);
+      __syncwarp();  // every lane's arrival is counted before lane 0's
+      if (lane == 0) mbar_expect_tx(full + slot, (unsigned)__popc(m) * (2 * D));
+      __syncwarp();
+      if (vr) bulk_g2s(row, vr, 2 * D, full + slot);
       issued = k + 1;
     };
     // Prologue: the first S tiles, each next row index already in flight.
@@ -2905,13 +2909,19 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       if (!mbar_wait(full + slot, (k / S) & 1)) { timed_out = true; break; }
       const uint32_t mask = mask_s[slot];
       const bool live = (mask >> lane) & 1u;
+      const float4 z4 = *reinterpret_cast<const float4*>(ring + slot * C::SLOT + lane * C::RP + 2 * D);
       float z[GM];
 #pragma unroll
-      for (int h = 0; h < GM; ++h) z[h] = (live && h < G) ? zs[(slot * GM + h) * 32 + lane] : -CUDART_INF_F;
+      for (int h = 0; h < GM; ++h) {
+        z[h] = -CUDART_INF_F;
+        if (live && h < G) {
+          if (h < 4) z[h] = h == 0 ? z4.x : h == 1 ? z4.y : h == 2 ? z4.z : z4.w;
+          else z[h] = zx[(slot * C::ZX + (h >= 4 ? h - 4 : 0)) * 32 + lane];
+        }
+      }
 
-      // Probabilities of this tile, written over its logits.
-      __syncwarp();
-      __nv_bfloat16* P = reinterpret_cast<__nv_bfloat16*>(zs + slot * GM * 32);
+      // Probabilities of this tile (the warp's buffer was last read by the
+      // previous tile's P.V, before the loop's closing __syncwarp).
 #pragma unroll
       for (int h = 0; h < GM; ++h) {
         if (h >= G) continue;
@@ -2938,7 +2948,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
 #pragma unroll
           for (int mi = 0; mi < C::MT; ++mi) {
             uint32_t a0, a1, a2, a3;
-            ldsm_x4_t(vt + swz_off<C::HALF_BYTES>(16 * sb + vrow, 16 * mi + vcol), a0, a1, a2, a3);
+            ldsm_x4_t(vt + (16 * sb + vrow) * C::RP + (16 * mi + vcol) * 2, a0, a1, a2, a3);
 #pragma unroll
             for (int nn = 0; nn < NT; ++nn) mma_bf16(acc[nn][mi], a0, a1, a2, a3, pb[nn][0], pb[nn][1]);
           }
@@ -2949,7 +2959,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
 #pragma unroll
         for (int mi = 0; mi < C::MT; ++mi) {
           uint32_t a0, a1, a2, a3;
-          ldsm_x4_t(vt + swz_off<C::HALF_BYTES>(16 * sb + vrow, 16 * mi + vcol), a0, a1, a2, a3);
+          ldsm_x4_t(vt + (16 * sb + vrow) * C::RP + (16 * mi + vcol) * 2, a0, a1, a2, a3);
           a0 &= mlo; a1 &= mlo; a2 &= mhi; a3 &= mhi;
 #pragma unroll
           for (int nn = 0; nn < NT; ++nn) mma_bf16(acc[nn][mi], a0, a1, a2, a3, pb[nn][0], pb[nn][1]);
