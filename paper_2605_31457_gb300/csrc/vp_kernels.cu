@@ -2802,6 +2802,8 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   const int64_t hrow0 = (int64_t)b * H + g * G;
   float (*tw)[kNsMax] = reinterpret_cast<float (*)[kNsMax]>(smem + C::OFF_TW);
   float (*tl)[kNsMax] = tw + GM;
+  // The sequence's record is a caller input: read it before the wait.
+  const Seq sq = load_seq(p, b, false);
   // (b) first: it reads only the score kernel's partials, complete before the
   // select kernel lets this grid start.  Its shared memory is the ring's.
   // After the anchor layer no select kernel runs in between: there (b)
@@ -2821,13 +2823,26 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   const int64_t pbase = ((int64_t)b * p.Hkv + g) * p.nk_max;
   unsigned err = 0;
   bool timed_out = false;
+  // The only CTA of its (sequence, kv-head) combines the text part with its
+  // chunk itself: no partial round trip through global memory, no ticket.
+  const bool lone = p.nc == 1 && p.nk == 1;
 
   // (a) kept chunk c
   if (c < p.nk) {
-    const Seq sq = load_seq(p, b, false);
     const int sel = p.granularity ? b * p.Hkv + g : b;
-    const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
+    // The first S + 1 tiles' kept indices are read in the same round trip
+    // as the count, at the chunk start a full list would give (exact for
+    // chunk 0 and whenever the count is the cap); entries past the count
+    // are masked below, a different start reloads them.
+    const int j0s = min(p.kept_cap, c * ((p.kept_cap + p.nk - 1) / p.nk));
+    int spec[S + 1];
+#pragma unroll
+    for (int k = 0; k <= S; ++k) {
+      const int j = j0s + 32 * (warp + kGmWarps * k) + lane;
+      spec[k] = j < p.kept_cap ? __ldcg(kept + j) : -1;
+    }
+    const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int per = (K + p.nk - 1) / p.nk;
     const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + C::MAX_CHUNK));
     if (per > C::MAX_CHUNK) err |= ERR_KEPT;  // the plan keeps every chunk within the limit
@@ -2848,6 +2863,17 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       }
       return i;
     };
+    // The same from a speculatively read entry (start j0s == j0).
+    auto spec_index = [&](int k, int raw) {
+      const int j = 32 * (warp + kGmWarps * k) + lane;
+      int i = -1;
+      if (k < nj && j0 + j < j1) {
+        i = raw;
+        if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
+      }
+      return i;
+    };
+    const bool spec_ok = j0 == j0s;
     auto issue = [&](int k, int i) {  // all lanes; i = this lane's kept index
       if (k >= nj) return;
       const int slot = k % S;
@@ -2877,11 +2903,11 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       issued = k + 1;
     };
     // Prologue: the first S tiles, each next row index already in flight.
-    int inext = row_index(0);
-#pragma unroll 1
+    int inext = spec_ok ? spec_index(0, spec[0]) : row_index(0);
+#pragma unroll
     for (int k = 0; k < S; ++k) {
       const int icur = inext;
-      inext = row_index(k + 1);
+      inext = spec_ok ? spec_index(k + 1, spec[k + 1]) : row_index(k + 1);
       issue(k, icur);
     }
     int ipend = inext;  // kept index for tile S (issued once tile 0 is read)
@@ -2983,6 +3009,25 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       const float l = warp_sum(lsum[h]);
       if (lane == 0) { wst[warp][h][0] = mh[h]; wst[warp][h][1] = l; }
     }
+    // Lone CTA: request the text output and statistics (the merged slice this
+    // CTA wrote in part (b), or the single split partial) before the sums.
+    constexpr int D4 = D / 4, IT = (GM * D4 + C::THREADS - 1) / C::THREADS;
+    float4 tv[IT];
+    float2 ts[IT];
+    if (lone) {
+      const float* t_o = p.nm ? p.mt_o + hrow0 * D : p.split_o + hrow0 * p.nsp_max * D;
+      const int t_ostride = p.nm ? D : p.nsp_max * D;
+#pragma unroll
+      for (int it = 0; it < IT; ++it) {
+        const int i = tid + it * C::THREADS;
+        if (i < G * D4) {
+          const int h = i / D4, d = 4 * (i % D4);
+          tv[it] = __ldcg(reinterpret_cast<const float4*>(t_o + (int64_t)h * t_ostride + d));
+          const float* st = p.nm ? p.mt_st + (hrow0 + h) * 2 : p.split_st + (hrow0 + h) * p.nsp_max * ST_N;
+          ts[it] = p.nm ? make_float2(__ldcg(st), __ldcg(st + 1)) : make_float2(__ldcg(st + ST_MT), __ldcg(st + ST_L1T));
+        }
+      }
+    }
     __syncthreads();  // every warp is done with its ring
     float* ow = reinterpret_cast<float*>(smem) + warp * GM * D;
 #pragma unroll
@@ -2996,7 +3041,34 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
         ow[(h0 + 1) * D + d0 + 8] = acc[nn][mi][3];
       }
     __syncthreads();
-    for (int i = tid; i < G * D; i += C::THREADS) {
+    if (lone) {
+      // Same arithmetic as the combine of gather_finish with one chunk.
+#pragma unroll
+      for (int it = 0; it < IT; ++it) {
+        const int i = tid + it * C::THREADS;
+        if (i >= G * D4) continue;
+        const int h = i / D4, d = 4 * (i % D4);
+        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+        float l = 0.f;
+#pragma unroll
+        for (int w = 0; w < kGmWarps; ++w) {
+          const float4 v = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(smem) + (w * GM + h) * D + d);
+          o.x += v.x; o.y += v.y; o.z += v.z; o.w += v.w;
+          l += wst[w][h][1];
+        }
+        const float mk = wst[0][h][0], mt = ts[it].x;
+        const float M = fmaxf(mt, mk);
+        const float wt = exp2_rel(mt, M), wk = exp2_rel(mk, M);
+        const float den = fmaf(wk, l, wt * ts[it].y);
+        const float inv = den > 0.f ? 1.f / den : 0.f;
+        float4 num = make_float4(wt * tv[it].x, wt * tv[it].y, wt * tv[it].z, wt * tv[it].w);
+        num.x = fmaf(wk, o.x, num.x); num.y = fmaf(wk, o.y, num.y); num.z = fmaf(wk, o.z, num.z); num.w = fmaf(wk, o.w, num.w);
+        __nv_bfloat16* op = reinterpret_cast<__nv_bfloat16*>(p.out) + (hrow0 + h) * D + d;
+        op[0] = from_f<__nv_bfloat16>(num.x * inv); op[1] = from_f<__nv_bfloat16>(num.y * inv);
+        op[2] = from_f<__nv_bfloat16>(num.z * inv); op[3] = from_f<__nv_bfloat16>(num.w * inv);
+      }
+    }
+    for (int i = tid; !lone && i < G * D; i += C::THREADS) {
       const int h = i / D, d = i % D;
       float o = 0.f, l = 0.f;
 #pragma unroll
@@ -3015,7 +3087,7 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
 
   if (timed_out) err |= ERR_TIMEOUT;
   if (err) atomicOr(p.err, err);
-  gather_finish<__nv_bfloat16, D, GM, C::THREADS>(p, b, g, hrow0, pbase, tw, fin, last);
+  if (!lone) gather_finish<__nv_bfloat16, D, GM, C::THREADS>(p, b, g, hrow0, pbase, tw, fin, last);
 }
 
 // ---------------------------------------------------------------------------
