@@ -201,6 +201,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity) {
     if (global_ns() - t0 > kWaitLimitNs) return false;
   }
 }
+// A 4-byte load through L2 issued where it stands in the program (the
+// compiler may not move it next to the value's first use), for prefetching.
+__device__ __forceinline__ int ldcg_now(const int* ptr) {
+  int v;
+  asm volatile("ld.global.cg.s32 %0, [%1];\n" : "=r"(v) : "l"(ptr));
+  return v;
+}
 // Orders this thread's earlier generic-proxy shared-memory accesses before
 // later asynchronous-proxy (bulk copy) writes to the same memory.
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
@@ -2831,17 +2838,22 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
   if (c < p.nk) {
     const int sel = p.granularity ? b * p.Hkv + g : b;
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
-    // The first S + 1 tiles' kept indices are read in the same round trip
-    // as the count, at the chunk start a full list would give (exact for
-    // chunk 0 and whenever the count is the cap); entries past the count
-    // are masked below, a different start reloads them.
+    // Kept-list entry of row `lane` of this warp's tile k for a chunk
+    // starting at j, read now (entries past the chunk are read in bounds
+    // and masked at use).  The copies of tile k are issued S tiles before it
+    // is consumed and its entry QD tiles before that: an iteration can take
+    // less than a round trip to L2.
+    constexpr int QD = 3;
+    auto raw_entry = [&](int j, int k) {
+      return ldcg_now(kept + min(j + 32 * (warp + kGmWarps * k) + lane, p.kept_cap - 1));
+    };
+    // The first S + QD tiles' entries are read in the same round trip as the
+    // count, at the chunk start a full list would give (exact for chunk 0
+    // and whenever the count is the cap); a different start reloads them.
     const int j0s = min(p.kept_cap, c * ((p.kept_cap + p.nk - 1) / p.nk));
-    int spec[S + 1];
+    int raw[S + QD];
 #pragma unroll
-    for (int k = 0; k <= S; ++k) {
-      const int j = j0s + 32 * (warp + kGmWarps * k) + lane;
-      spec[k] = j < p.kept_cap ? __ldcg(kept + j) : -1;
-    }
+    for (int k = 0; k < S + QD; ++k) raw[k] = raw_entry(j0s, k);
     const int K = max(0, min(__ldcg(p.kept_count + sel), min(sq.nv, p.kept_cap)));
     const int per = (K + p.nk - 1) / p.nk;
     const int j0 = min(K, c * per), j1 = min(K, min(j0 + per, j0 + C::MAX_CHUNK));
@@ -2851,29 +2863,21 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
     const float* zb = p.z_ws + (int64_t)b * p.max_visual * p.hp + g * G;
     int issued = 0;  // tiles of this warp whose copies were issued
 
-    // Kept index of row `lane` of this warp's tile k, or -1 (read from the
-    // kept list a tile ahead of its copies; an out-of-range index is
-    // flagged and skipped).
-    auto row_index = [&](int k) {
+    // Kept index of row `lane` of this warp's tile k from its entry, or -1
+    // (past the chunk; an out-of-range index is flagged and skipped).
+    auto row_index = [&](int k, int e) {
       const int j = 32 * (warp + kGmWarps * k) + lane;
       int i = -1;
       if (k < nj && j0 + j < j1) {
-        i = __ldcg(kept + j0 + j);
+        i = e;
         if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
       }
       return i;
     };
-    // The same from a speculatively read entry (start j0s == j0).
-    auto spec_index = [&](int k, int raw) {
-      const int j = 32 * (warp + kGmWarps * k) + lane;
-      int i = -1;
-      if (k < nj && j0 + j < j1) {
-        i = raw;
-        if (i < 0 || i >= sq.nv) { err |= ERR_KEPT; i = -1; }
-      }
-      return i;
-    };
-    const bool spec_ok = j0 == j0s;
+    if (j0 != j0s) {  // CTA-uniform
+#pragma unroll
+      for (int k = 0; k < S + QD; ++k) raw[k] = raw_entry(j0, k);
+    }
     auto issue = [&](int k, int i) {  // all lanes; i = this lane's kept index
       if (k >= nj) return;
       const int slot = k % S;
@@ -2902,15 +2906,12 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
       if (vr) bulk_g2s(row, vr, 2 * D, full + slot);
       issued = k + 1;
     };
-    // Prologue: the first S tiles, each next row index already in flight.
-    int inext = spec_ok ? spec_index(0, spec[0]) : row_index(0);
+    // Prologue: the first S tiles; the next QD tiles' entries stay queued.
 #pragma unroll
-    for (int k = 0; k < S; ++k) {
-      const int icur = inext;
-      inext = spec_ok ? spec_index(k + 1, spec[k + 1]) : row_index(k + 1);
-      issue(k, icur);
-    }
-    int ipend = inext;  // kept index for tile S (issued once tile 0 is read)
+    for (int k = 0; k < S; ++k) issue(k, row_index(k, raw[k]));
+    int q[QD];
+#pragma unroll
+    for (int t = 0; t < QD; ++t) q[t] = raw[S + t];
 
     // Probabilities are taken relative to each head's largest logit over all
     // tokens (from the select kernel), so no running maximum is needed.
@@ -2992,9 +2993,11 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
         }
       }
       __syncwarp();
-      // Refill this slot with tile k + S.
-      const int icur = ipend;
-      ipend = row_index(k + S + 1);
+      // Refill this slot with tile k + S; queue the entry of tile k + S + QD.
+      const int icur = row_index(k + S, q[0]);
+#pragma unroll
+      for (int t = 0; t + 1 < QD; ++t) q[t] = q[t + 1];
+      q[QD - 1] = raw_entry(j0, k + S + QD);
       issue(k + S, icur);
     }
     // After a timeout, let this warp's copies still in flight land (bounded)
