@@ -218,19 +218,15 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, unsigned by
 
 // 16- and 4-byte asynchronous copies global -> shared (LSU path), and the
 // arrive-on that completes an mbarrier phase once this thread's earlier such
-// copies have landed (the barrier's count must include these arrivals).
+// copies have landed; the barrier's pending count is raised first, so the
+// arrival needs no room in the barrier's count (a normal arrival still
+// completes the phase once the copies have landed).
 __device__ __forceinline__ void cp_async16(unsigned dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_async4(unsigned dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
 }
-__device__ __forceinline__ void cp_async_arrive(uint64_t* bar) {
-  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];\n" ::"r"(smem_u32(bar)) : "memory");
-}
-// The same arrive-on, but the barrier's pending count is raised first, so
-// the arrival needs no room in the barrier's count (a normal arrival still
-// completes the phase once the copies have landed).
 __device__ __forceinline__ void cp_async_arrive_counted(uint64_t* bar) {
   asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];\n" ::"r"(smem_u32(bar)) : "memory");
 }
@@ -2738,16 +2734,18 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(const __grid_constant
 // padded rows (a 16-byte shift per row: conflict-free ldmatrix), and the
 // token's logits with 4-byte cp.async (heads 0-3 into the row's pad bytes);
 // the slot's mbarrier completes once the row bytes and every lane's logits
-// have landed.  The kept indices are read from the kept list one tile ahead
-// of their copies.  S is 1 when no chunk holds more than one tile per warp (four CTAs
-// share an SM); otherwise 3 (two CTAs per SM) or 2 (three CTAs per SM,
-// the same bytes in flight per SM over more warps), whichever runs the grid
-// in fewer waves, 3 on a tie (a lone CTA in a short last wave keeps more
-// copies in flight).  The tile's logits give per-head probabilities; P.V
-// runs on the tensor cores as in the score kernel (A = V^T by
-// ldmatrix.trans, B = P^T from a per-warp bf16 buffer).  The warps'
-// partials are merged into the chunk's partial; (b) and the final combine
-// are shared with k_gather.
+// have landed.  The kept-list entries are read three tiles ahead of their
+// copies (the first ones in the same round trip as the kept count).  S is 1
+// when no chunk holds more than one tile per warp (four CTAs share an SM);
+// otherwise 3 (two CTAs per SM) or 2 (three CTAs per SM, the same bytes in
+// flight per SM over more warps), whichever runs the grid in fewer waves, 3
+// on a tie (a lone CTA in a short last wave keeps more copies in flight).
+// The tile's logits give per-head probabilities; P.V runs on the tensor
+// cores as in the score kernel (A = V^T by ldmatrix.trans, B = P^T from a
+// per-warp bf16 buffer).  The warps' partials are merged in shared memory:
+// the only CTA of its (sequence, kv-head) combines them with the text part
+// and writes the output; otherwise they form the chunk's partial, and (b)
+// and the final combine are shared with k_gather.
 // ---------------------------------------------------------------------------
 constexpr int kGmWarps = 4;
 constexpr int kGmSlots = 3;  // ring slots of the deeper form (the other has 2)
