@@ -4,8 +4,10 @@
 // every sequence's tiles for the tensor-core kernel within the page-id
 // staging bound, keeps every gather chunk within the chunk kernel's limit and
 // picks the slice gather only for kept sets it holds; a table of call shapes
-// gets its expected select form.  Prints one line per violation and exits
-// non-zero if there was any.
+// gets its expected select form, and a table of the chunk gather's call
+// shapes its chunk count, CTAs per (sequence, kv-head) and whether the lone
+// CTA combines in place.  Prints one line per violation and exits non-zero if
+// there was any.
 #include <cstdio>
 
 #include "vp_internal.h"
@@ -63,6 +65,43 @@ int check_forms() {
     if (kind != c.want_kind || w != c.want_w) {
       std::printf("FAIL select form of %s: kind %d (want %d), slice %d (want %d), cluster %d\n", c.name, kind,
                   c.want_kind, w, c.want_w, pl.cl);
+      ++bad;
+    }
+  }
+  return bad;
+}
+
+// Chunk-gather plans of the benchmarked sweep shapes (B = 64, 32/8 heads,
+// D = 128, 1024 text tokens; fixed ratios 5% / 20% / 50% and top-p, whose
+// cap is the whole span) and of the dense layers of the anchor pipeline: the
+// GPU parity tests at these sizes run every combine form through them.
+struct ChunkCase {
+  const char* name;
+  int B, Hkv, D, max_visual, max_seq, kept_cap, tc;
+  int want_nk, want_nm, want_nc;
+};
+
+int check_chunks() {
+  using namespace vp;
+  const int T = 1024 + 18;
+  const ChunkCase cases[] = {
+      // name, B, Hkv, D, N_v, max_seq, kept_cap, tc, nk, nm, nc
+      {"sweep N_v 576, 50% (one score split: text from its partial)", 64, 8, 128, 576, 576 + T, 288, 0, 1, 0, 1},
+      {"sweep N_v 2304, 50%", 64, 8, 128, 2304, 2304 + T, 1152, 1, 1, 0, 1},
+      {"sweep N_v 6400, 20%", 64, 8, 128, 6400, 6400 + T, 1280, 1, 1, 0, 1},
+      {"sweep N_v 6400, 50% (two chunks, text from the split partial)", 64, 8, 128, 6400, 6400 + T, 3200, 1, 2, 0, 2},
+      {"sweep N_v 16384, 5% (lone CTA, merged text slice)", 64, 8, 128, 16384, 16384 + T, 820, 1, 1, 1, 1},
+      {"sweep N_v 16384, 20%", 64, 8, 128, 16384, 16384 + T, 3277, 1, 2, 2, 2},
+      {"sweep N_v 16384, 50%", 64, 8, 128, 16384, 16384 + T, 8192, 1, 4, 4, 4},
+      {"sweep N_v 16384, top-p (cap = span, chunk starts differ)", 64, 8, 128, 16384, 16384 + T, 16384, 1, 8, 8, 8},
+      {"dense layer of the anchor pipeline, B = 1", 1, 4, 128, 1296, 4113, 1296, 0, 6, 4, 6},
+  };
+  int bad = 0;
+  for (const ChunkCase& c : cases) {
+    const Plan pl = make_plan(c.B, c.Hkv, c.D, 152, c.max_visual, c.max_seq, c.kept_cap, 0, c.tc != 0);
+    if (pl.gslice || pl.nk != c.want_nk || pl.nm != c.want_nm || pl.nc != c.want_nc) {
+      std::printf("FAIL chunk plan of %s: nk %d nm %d nc %d gslice %d (want %d %d %d 0)\n", c.name, pl.nk, pl.nm,
+                  pl.nc, pl.gslice, c.want_nk, c.want_nm, c.want_nc);
       ++bad;
     }
   }
@@ -136,5 +175,6 @@ int main() {
             }
   std::printf("%lld plans, %d violations\n", plans, fails);
   fails += check_forms();
+  fails += check_chunks();
   return fails ? 1 : 0;
 }

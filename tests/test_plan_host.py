@@ -3,9 +3,11 @@ run on the CPU (no GPU): score splits cover the whole cache and fit the
 workspace, the tensor-core kernel's weighted splits partition every
 sequence's tiles within the page-id staging bound, gather chunks stay within
 the chunk kernel's limit, the slice gather is chosen only for kept sets it
-can hold, and every benchmarked call shape gets the expected select form
+can hold, every benchmarked call shape gets the expected select form
 (fused select + gather and its slice width, select only, or the
-shared-memory select) (tests/plan_invariants.cpp)."""
+shared-memory select), and the chunk gather's benchmarked shapes get their
+expected chunk count, text-merge slices and CTAs per (sequence, kv-head)
+(tests/plan_invariants.cpp)."""
 
 import os
 import shutil
