@@ -2838,12 +2838,13 @@ __global__ void __launch_bounds__(32 * kGmWarps) k_gather_mma(const __grid_const
     const int32_t* kept = p.kept_idx + (int64_t)sel * p.kept_cap;
     // Kept-list entry of row `lane` of this warp's tile k for a chunk
     // starting at j, read now (entries past the chunk are read in bounds
-    // and masked at use).  The copies of tile k are issued S tiles before it
+    // and masked at use; with no kept capacity the list may be absent and
+    // nothing is read).  The copies of tile k are issued S tiles before it
     // is consumed and its entry QD tiles before that: an iteration can take
     // less than a round trip to L2.
     constexpr int QD = 3;
     auto raw_entry = [&](int j, int k) {
-      return ldcg_now(kept + min(j + 32 * (warp + kGmWarps * k) + lane, p.kept_cap - 1));
+      return p.kept_cap > 0 ? ldcg_now(kept + min(j + 32 * (warp + kGmWarps * k) + lane, p.kept_cap - 1)) : -1;
     };
     // The first S + QD tiles' entries are read in the same round trip as the
     // count, at the chunk start a full list would give (exact for chunk 0

@@ -152,6 +152,37 @@ def test_chunk_gather_paths(vp, dtype, D, batch, budget, heads):
     Hn.check_all(vp, Hn.make_inputs(r), budget)
 
 
+def test_zero_kept_capacity_on_the_chunk_gather(vp):
+    """A budget that keeps nothing (fixed K = 0: kept capacity 0 and no kept
+    array at all) on a shape that takes the shared-memory select and the
+    chunk gather (16 sequences x 4 kv-heads, more than 4096 visual tokens):
+    nothing is read from the absent list, and the output is the attention
+    over the text tokens alone."""
+    budget = dict(mode=O.FIXED_K, tau=0.1, fixed_k=0)
+    B = 16
+    rng = np.random.default_rng(B)
+    vis = tuple(int(x) for x in rng.integers(4097, 4200, B))
+    start = tuple(int(x) for x in rng.integers(0, 40, B))
+    text = tuple(int(s) + int(x) for s, x in zip(start, rng.integers(1, 200, B)))
+    inp = Hn.make_inputs(small(batch=B, vis_len=vis, vis_start=start, text_len=text))
+    dev = Hn.Device(vp, inp, budget)
+    try:
+        assert vp.vp_max_kept(dev.budget, dev.cfg.max_visual) == 0
+        vp.vp_decode_step(dev.ctx, B, dev.q, dev.kc, dev.vc, dev.span, dev.tl, dev.budget, dev.out, None, 0,
+                          dev.count, dev.mass, dev.stats)
+        vp.vp_check_errors(dev.ctx)
+        assert vp.vp_last_launch(dev.ctx)[1] == 3, "score, select and chunk gather should serve this batch"
+        torch.cuda.synchronize()
+        gpu = dict(out=dev.out.float().cpu().numpy(), kept=np.full((B, 1, 1), -1, np.int32),
+                   count=dev.count.cpu().numpy().reshape(B, 1), mass=dev.mass.cpu().numpy(),
+                   stats=dev.stats.cpu().numpy())
+        assert np.all(gpu["count"] == 0)
+        for b in (0, 7, 15):
+            Hn.compare_seq(inp, gpu, b, budget)
+    finally:
+        dev.close()
+
+
 def test_explicit_logit_scale(vp):
     r = small()
     Hn.check_all(vp, Hn.make_inputs(r), dict(r.budget, scale=0.05))
